@@ -1,0 +1,463 @@
+"""Benchmark of the BRISK-DLM per-block decode tail on GB300.
+
+A step is one fused decode-tail call (candidates + corrector + verification)
+over one block of the decode-stream workload: 128 sequences, block length 32,
+vocabulary 126464, width 4096, K = 8, corrector width 256, bf16 logits and
+hidden states, greedy Select and verify, per-sequence verifier agreement
+U(0.6, 0.98). The timed steps cycle through a pool of distinct pre-generated
+blocks (each block's 2.07 GB of logits exceeds the 129 MB L2, so no flush is
+needed); the anchor of each block is the last committed token of the block
+before it. The metric is accepted (verified) tokens per second.
+
+Under torchrun every rank runs its own 128 sequences (replicas: the method
+has no exchange between sequences); the value is the accepted tokens of all
+ranks over the slowest rank's time.
+
+``--impl reference`` times the CPU oracle (the plain float64 statement of the
+method) on a bounded sample of the same workload instead.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "verified tokens/sec at 1 GB300 for decode tail; % of HBM roofline on vocab sweep"
+UNIT = "accepted tokens/s"
+WORKLOAD = "decode_stream"
+NAMEPLATE_HBM_GBS = 8000.0
+FALLBACK_HBM_GBS = 6800.0
+SWEEP_KERNEL_SRC = os.path.join(ROOT, "paper_2609_33390_gb300", "csrc", "sweep.cu")
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "ncu_traffic.txt")
+
+
+# ----------------------------------------------------------------------------- host helpers
+
+def dist_env():
+    return (int(os.environ.get("RANK", "0")), int(os.environ.get("WORLD_SIZE", "1")),
+            int(os.environ.get("LOCAL_RANK", "0")))
+
+
+def shard_sequences(rank: int, world: int, per_rank: int, n_seqs: int):
+    """Sequence ids of one rank: ranks take consecutive groups of `per_rank` sequences of the
+    stream, wrapping around its `n_seqs` sequences."""
+    start = (rank * per_rank) % max(1, n_seqs)
+    return [(start + j) % n_seqs for j in range(per_rank)]
+
+
+def aggregate(total_tokens_local: float, elapsed_local_s: float, reduce_sum, reduce_max):
+    """Whole-job throughput: tokens of every rank over the slowest rank's time."""
+    tokens = reduce_sum(total_tokens_local)
+    elapsed = reduce_max(elapsed_local_s)
+    return tokens / elapsed, tokens, elapsed
+
+
+def measured_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    return FALLBACK_HBM_GBS, "fallback"
+
+
+def sweep_source_hash() -> str:
+    with open(SWEEP_KERNEL_SRC, "rb") as f:
+        return hashlib.sha1(f.read()).hexdigest()[:12]
+
+
+def recorded_traffic(workload: str):
+    """DRAM bytes per sweep launch from the committed ncu summary, when it was taken on the
+    current sweep source (lines: kernel workload bytes_per_launch source_hash)."""
+    if not os.path.exists(TRAFFIC_FILE):
+        return None
+    h = sweep_source_hash()
+    with open(TRAFFIC_FILE) as f:
+        for line in f:
+            parts = line.split()
+            if len(parts) >= 4 and parts[0] == "sweep" and parts[1] == workload and parts[3] == h:
+                return float(parts[2])
+    return None
+
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons during the timed region."""
+    QUERY = ("timestamp,index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.lines = []
+        self.t = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.QUERY}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except (FileNotFoundError, OSError):
+            self.proc = None
+            return
+        self.t = threading.Thread(target=self._read, daemon=True)
+        self.t.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append((time.time(), line.strip()))
+
+    def stop(self):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+        if self.t is not None:
+            self.t.join(timeout=2)
+
+    def summary(self, t0: float, t1: float):
+        rows = []
+        for ts, line in self.lines:
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 10:
+                continue
+            try:
+                rows.append((ts, float(parts[2]), float(parts[3]), parts[5:]))
+            except ValueError:
+                continue
+        inside = [r for r in rows if t0 <= r[0] <= t1 + 0.15]
+        used = inside if inside else rows
+        if not used:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no nvidia-smi samples"],
+                    "samples": 0}
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = set()
+        for r in used:
+            for n, v in zip(names, r[3][1:5]):
+                if v.strip().lower() == "active":
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(r[1] for r in used),
+                "sm_max_mhz": max(r[2] for r in used), "reasons": sorted(reasons),
+                "samples": len(used), "samples_in_timed_region": len(inside)}
+
+
+# ----------------------------------------------------------------------------- CPU oracle leg
+
+CPU_SAMPLE_SEQS = 8
+
+
+def _oracle_sample_worker(spec_json: str) -> str:
+    """Runs in a fresh single-threaded interpreter: generates a bounded sample of the workload on
+    the CPU and times the oracle's decode tail on it."""
+    spec = json.loads(spec_json)
+    import numpy as np
+    import torch
+    torch.set_num_threads(1)
+    from paper_2609_33390_gb300 import synth
+    from oracle import brisk_oracle as O
+    wl = synth.WORKLOADS[spec["workload"]]
+    seqs = spec["seqs"]
+    block = synth.make_block(wl, "cpu", seqs=seqs, block=spec["block"])
+    # corrector weights (small) and on-demand embedding rows of the full vocabulary
+    ws = {k: v.to(torch.float64).numpy()
+          for k, v in synth.make_corrector_weights(wl, "cpu").items()}
+    gen_time = [0.0]
+
+    class Rows:
+        def __init__(self, which):
+            self.src = synth.EmbeddingRows(wl, which)
+            self.cache = {}
+
+        def __getitem__(self, v):
+            v = int(v)
+            if v not in self.cache:
+                t = time.perf_counter()
+                self.cache[v] = self.src[v].to(torch.float64).numpy()
+                gen_time[0] += time.perf_counter() - t
+            return self.cache[v]
+
+    ws.update(E_in=Rows("E_in"), E_out=Rows("E_out"), b_g=0.0, alpha=0.0)
+    params = O.params_from_arrays(ws)
+    lq = block["logits_q"].to(torch.float64).numpy()
+    lp = block["logits_p"].to(torch.float64).numpy()
+    hid = block["hidden"].to(torch.float64).numpy()
+    hc = block["h_c"].to(torch.float64).numpy()
+    x0 = block["x0"].numpy()
+    t0 = time.perf_counter()
+    acc = 0
+    for b in range(len(seqs)):
+        _, _, _, _, vr = O.decode_tail_sequence(params, lambda i: lq[b, i], lambda i: lp[b, i],
+                                                hid[b], hc[b], int(x0[b]), wl.K, wl.select_mode,
+                                                wl.verify_mode)
+        acc += vr.accepted_len
+    el = time.perf_counter() - t0 - gen_time[0]
+    return json.dumps({"accepted": acc, "seconds": el, "seqs": len(seqs)})
+
+
+def run_oracle_sample(seqs, block=0, workload=WORKLOAD):
+    env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1",
+               CUDA_VISIBLE_DEVICES="")
+    spec = json.dumps({"workload": workload, "seqs": list(seqs), "block": block})
+    code = ("import sys; sys.path.insert(0, %r); import bench; print(bench._oracle_sample_worker(%r))"
+            % (ROOT, spec))
+    r = subprocess.run([sys.executable, "-c", code], env=env, capture_output=True, text=True,
+                       cwd=ROOT)
+    if r.returncode != 0:
+        raise RuntimeError("oracle sample failed:\n" + r.stderr[-2000:])
+    return json.loads(r.stdout.strip().splitlines()[-1])
+
+
+def cpu_baseline_entry(seqs):
+    res = run_oracle_sample(seqs)
+    return {"value": res["accepted"] / res["seconds"], "unit": UNIT, "cores": 1, "kind": "oracle",
+            "sample": f"{res['seqs']} sequences x 1 block of {WORKLOAD} (L=32, V=126464, d=4096,"
+                      f" K=8, r=256), float64 numpy oracle, {res['seconds']:.1f} s of CPU time"}
+
+
+# ----------------------------------------------------------------------------- reference arm
+
+def run_reference(args):
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return 0
+    from paper_2609_33390_gb300 import synth
+    wl = synth.WORKLOADS[WORKLOAD]
+    per_step = 1
+    for w in range(args.warmup):
+        run_oracle_sample([w % wl.n_seqs], block=0)
+    tot_acc, tot_s = 0, 0.0
+    for s in range(args.steps):
+        r = run_oracle_sample([(s * per_step) % wl.n_seqs], block=s % wl.n_blocks)
+        tot_acc += r["accepted"]
+        tot_s += r["seconds"]
+    value = tot_acc / tot_s
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000.0 * tot_s / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic",
+        "config": {"workload": WORKLOAD, "B": 1, "L": wl.L, "V": wl.V, "d": wl.d, "K": wl.K,
+                   "r": wl.r, "step": "one sequence of one block per step"},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
+                         "sample": "one sequence of the decode-stream workload per step"},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line))
+    return 0
+
+
+# ----------------------------------------------------------------------------- GPU arm
+
+def run_ours(args):
+    import torch
+    from paper_2609_33390_gb300 import build, brisk, synth
+
+    rank, world, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    build.build()
+    wl = synth.WORKLOADS[WORKLOAD]
+    seqs = shard_sequences(rank, world, wl.B, wl.n_seqs)
+
+    weights = synth.make_weights(wl, dev)
+    tail = brisk.DecodeTail.for_workload(wl, weights, dev)
+    t = time.perf_counter()
+    tail.prepare()
+    torch.cuda.synchronize()
+    prepare_ms = 1000.0 * (time.perf_counter() - t)
+
+    pool_n = max(1, min(args.pool, args.steps + args.warmup))
+    pool = []
+    for j in range(pool_n):
+        blk = synth.make_block(wl, dev, seqs=seqs, block=j % wl.n_blocks)
+        pool.append(blk)
+    sm, vm = brisk.mode_ids(wl.select_mode, wl.verify_mode)
+    nsteps = args.warmup + args.steps
+    outs = [tail.alloc_outputs(full=False) for _ in range(nsteps)]
+    events = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+              for _ in range(nsteps)]
+    stream = torch.cuda.current_stream()
+    for e0, e1 in events:      # create the CUDA events before handing their handles over
+        e0.record(stream)
+        e1.record(stream)
+    torch.cuda.synchronize()
+
+    def step(s):
+        blk = pool[s % pool_n]
+        x0 = blk["x0"] if s == 0 else outs[s - 1]["next_anchor"]
+        tail.tail(blk, sm, vm, out=outs[s], x0=x0, events=events[s])
+
+    sampler = ClockSampler(local if "CUDA_VISIBLE_DEVICES" not in os.environ else 0)
+    sampler.start()
+    time.sleep(0.3)
+    for s in range(args.warmup):
+        step(s)
+    torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    g0 = torch.cuda.Event(enable_timing=True)
+    g1 = torch.cuda.Event(enable_timing=True)
+    wall0 = time.time()
+    g0.record(stream)
+    for s in range(args.warmup, nsteps):
+        step(s)
+    g1.record(stream)
+    torch.cuda.synchronize()
+    wall1 = time.time()
+    if world > 1:
+        torch.distributed.barrier()
+    time.sleep(0.25)
+    sampler.stop()
+    elapsed = g0.elapsed_time(g1) / 1000.0
+    status = tail.device_status()
+    if status != brisk.OK:
+        raise RuntimeError(f"device status {brisk.status_string(status)}")
+
+    acc = sum(int(outs[s]["accepted_len"].sum()) for s in range(args.warmup, nsteps))
+    committed = sum(int((outs[s]["accepted_len"] + (outs[s]["correction"] >= 0).int()).sum())
+                    for s in range(args.warmup, nsteps))
+    sweep_ms = [events[s][0].elapsed_time(events[s][1]) for s in range(args.warmup, nsteps)]
+
+    if world > 1:
+        import torch.distributed as dist
+
+        def rsum(x):
+            t_ = torch.tensor([float(x)], device=dev, dtype=torch.float64)
+            dist.all_reduce(t_, op=dist.ReduceOp.SUM)
+            return float(t_.item())
+
+        def rmax(x):
+            t_ = torch.tensor([float(x)], device=dev, dtype=torch.float64)
+            dist.all_reduce(t_, op=dist.ReduceOp.MAX)
+            return float(t_.item())
+    else:
+        rsum = rmax = float
+    value, tokens, elapsed_max = aggregate(acc, elapsed, rsum, rmax)
+    committed_all = rsum(committed)
+
+    # roofline of the dominant kernel (the vocabulary sweep)
+    sweep_bytes = wl.sweep_bytes()
+    mean_sweep_s = statistics.mean(sweep_ms) / 1000.0
+    achieved = sweep_bytes / mean_sweep_s / 1e9
+    peak, peak_src = measured_peaks()
+    traffic = recorded_traffic(WORKLOAD)
+
+    # end to end through the public API: inputs from pinned host memory every step
+    e2e = run_e2e(args, tail, pool, wl, sm, vm, dev) if rank == 0 or world > 1 else None
+    if world > 1 and e2e is not None:
+        e2e["value"] = rsum(e2e["_tokens"]) / rmax(e2e["_seconds"])
+    if e2e is not None:
+        e2e.pop("_tokens", None)
+        e2e.pop("_seconds", None)
+
+    if rank != 0:
+        return 0
+    cpu = None
+    if not args.no_cpu_baseline:
+        cpu = cpu_baseline_entry(list(range(CPU_SAMPLE_SEQS)))
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": 1000.0 * elapsed_max / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+        "data": "synthetic",
+        "config": {"workload": WORKLOAD, "B": wl.B, "L": wl.L, "V": wl.V, "d": wl.d, "K": wl.K,
+                   "r": wl.r, "input_dtype": "bf16", "select": wl.select_mode,
+                   "verify": wl.verify_mode, "parallelism": "replicas",
+                   "l2": f"inputs larger than L2 ({sweep_bytes / 1e9:.2f} GB of logits per step,"
+                         f" {pool_n} distinct blocks cycled)",
+                   "prepare_ms": round(prepare_ms, 1)},
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                     "frac": achieved / peak, "traffic": traffic, "peak_source": peak_src,
+                     "kernel": "sweep_kernel (proposal + verifier rows)",
+                     "bytes_per_launch": sweep_bytes, "mean_launch_us": 1e6 * mean_sweep_s,
+                     "frac_of_nameplate_8tbs": achieved / NAMEPLATE_HBM_GBS},
+        "cpu_baseline": cpu,
+        "e2e": e2e,
+        "gpu_launches": brisk.kernels_per_tail(tail.dims) * args.steps,
+        "clocks": sampler.summary(wall0, wall1),
+        "committed_tokens_per_s": committed_all / elapsed_max,
+        "accepted_per_sequence_block": tokens / (wl.B * world * args.steps),
+    }
+    print(json.dumps(line))
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+    return 0
+
+
+def run_e2e(args, tail, pool, wl, sm, vm, dev):
+    """Same metric through the public API with host buffers: every step copies the block's
+    inputs from pinned host memory and reads the accepted lengths and tokens back."""
+    import torch
+    n = max(1, min(args.e2e_steps, args.steps))
+    keys = ("logits_q", "logits_p", "hidden", "h_c", "x0")
+    host = []
+    for j in range(min(2, len(pool))):
+        host.append({k: pool[j][k].cpu().pin_memory() for k in keys})
+    dev_in = {k: torch.empty_like(pool[0][k]) for k in keys}
+    out = tail.alloc_outputs(full=False)
+    res_host = {k: torch.empty(out[k].shape, dtype=out[k].dtype).pin_memory()
+                for k in ("accepted_len", "out_tokens", "correction")}
+    h2d = sum(host[0][k].numel() * host[0][k].element_size() for k in keys)
+    d2h = sum(v.numel() * v.element_size() for v in res_host.values())
+    stream = torch.cuda.current_stream()
+    torch.cuda.synchronize()
+    acc = 0
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    for it in range(n + 1):
+        if it == 1:
+            torch.cuda.synchronize()
+            acc = 0
+            e0.record(stream)
+        h = host[it % len(host)]
+        for k in keys:
+            dev_in[k].copy_(h[k], non_blocking=True)
+        tail.tail(dev_in, sm, vm, out=out)
+        for k, v in res_host.items():
+            v.copy_(out[k], non_blocking=True)
+        stream.synchronize()
+        if it >= 1:
+            acc += int(res_host["accepted_len"].sum())
+    e1.record(stream)
+    torch.cuda.synchronize()
+    secs = e0.elapsed_time(e1) / 1000.0
+    return {"value": acc / secs, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+            "steps": n, "ms_per_step": 1000.0 * secs / n, "_tokens": acc, "_seconds": secs}
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__.splitlines()[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=400)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--pool", type=int, default=16, help="distinct pre-generated blocks cycled")
+    ap.add_argument("--e2e-steps", type=int, default=20)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args(argv)
+    args.warmup = max(3, args.warmup)   # at least 3 untimed warm-up steps
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_ours(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,205 @@
+/*
+ * brisk.h - C ABI of the BRISK-DLM per-block decode tail on GB300 (sm_103a).
+ *
+ * The decode tail turns one backbone evaluation of a diffusion language model
+ * into verified tokens (paper: "From Position Risks to Block Survival: Faster
+ * Generation for Diffusion Language Models", Sec. 3.3 and Algorithm 1(b)):
+ *
+ *   1. candidates: log-sum-exp over the full vocabulary and the ordered Top-K
+ *      of every masked position (Sec. 3.3 "C_i = TopK(q_i, K)"; App. C.2);
+ *   2. the prefix-conditioned corrector, which reranks only those K
+ *      candidates with a minimal-GRU state that reads the tokens selected
+ *      earlier in the block (Sec. 3.3 Eqs. 4-5; App. C.2 Eq. 7);
+ *   3. left-to-right verification against the verifier distribution up to the
+ *      first rejection (Sec. 3.1; Sec. 3.3; App. B Eq. 8).
+ *
+ * Conventions shared by every entry point:
+ *  - Every tensor argument is caller-owned device memory, row-major and dense
+ *    (the last dimension contiguous). The library never allocates or frees
+ *    device memory; scratch lives in a caller-provided workspace of
+ *    brisk_workspace_bytes() bytes and the folded corrector tables in a
+ *    caller-provided buffer of brisk_tables_bytes() bytes, both 256-byte
+ *    aligned. A workspace must not be shared by calls that may overlap; its
+ *    contents need no initialisation.
+ *  - `stream` is a cudaStream_t passed as void* (NULL = legacy default
+ *    stream). Calls only enqueue work and return; results are ready when the
+ *    stream reaches them. Every call may be captured into a CUDA graph.
+ *  - Host-detectable problems (NULL pointers, unsupported sizes, bad modes,
+ *    misaligned buffers) return an error before anything is enqueued. A
+ *    failed kernel launch returns BRISK_ERR_CUDA. Problems found on the
+ *    device are recorded in a status word in the workspace, read with
+ *    brisk_last_device_status(); the first one of a call wins.
+ *  - Logit and hidden tensors are fp32 or bf16 as the dims say; every
+ *    internal sum and score is fp32. Ids are int32.
+ *  - Positions are 0-based: position i of the block is the paper's i+1, and
+ *    the token before position 0 is the anchor x0 (the paper's x_0).
+ */
+#ifndef BRISK_H
+#define BRISK_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum brisk_status {
+  BRISK_OK = 0,
+  BRISK_ERR_INVALID_ARG = 1,   /* NULL pointer, bad mode, size out of range, misaligned buffer */
+  BRISK_ERR_UNSUPPORTED = 2,   /* valid request this build does not implement                   */
+  BRISK_ERR_CUDA = 3,          /* a CUDA call or kernel launch failed                           */
+  BRISK_ERR_TIMEOUT = 4,       /* a bounded device-side wait gave up                            */
+  BRISK_ERR_NUMERIC = 5        /* a row's log-partition was not finite (NaN / all -inf)          */
+} brisk_status;
+
+typedef enum brisk_dtype { BRISK_DT_F32 = 0, BRISK_DT_BF16 = 1 } brisk_dtype;
+
+/* Select rule of Algorithm 1(b): argmax of the refined scores (lowest rank on ties),
+ * or one draw from softmax of the refined scores with a caller uniform. */
+typedef enum brisk_select_mode { BRISK_SELECT_GREEDY = 0, BRISK_SELECT_SAMPLE = 1 } brisk_select_mode;
+
+/* Verification: greedy (accept iff x_i is the verifier argmax) or speculative sampling
+ * (accept iff u < min(1, p_i(x_i)/pi_i(x_i)), resample from [p_i - pi_i]_+; Sec. 3.3). */
+typedef enum brisk_verify_mode { BRISK_VERIFY_GREEDY = 0, BRISK_VERIFY_STOCHASTIC = 1 } brisk_verify_mode;
+
+/* Problem sizes. B sequences, block length L (the paper's M), vocabulary V, backbone width d,
+ * K candidates, corrector width r. The corrector state has S = 2r dimensions; the position
+ * embedding and the feature projection have 16 (App. C.2 head configuration, with
+ * rank = hidden projection = token projection = r).
+ * Limits: B >= 1; 1 <= L <= 64; 4 <= K <= 32; V >= K; d >= 8 and d % 8 == 0;
+ * 16 <= r <= 512 and r % 16 == 0. */
+typedef struct brisk_dims {
+  int32_t B, L, V, d, K, r;
+  int32_t logits_dtype;   /* brisk_dtype of logits_q / logits_p                        */
+  int32_t hidden_dtype;   /* brisk_dtype of hidden, h_ctx, every weight and E_in/E_out */
+} brisk_dims;
+
+/* Corrector parameters psi and the frozen vocabulary rows (App. C.2), device pointers in
+ * hidden_dtype, row-major:
+ *   E_in  [V, d]   frozen input token embedding E
+ *   E_out [V, d]   frozen LM-head rows E_out
+ *   P_h   [r, d]   projection of MASK hidden states and of h_ctx
+ *   P_e   [r, d]   projection of token embeddings
+ *   P_phi [16, 5]  projection of the 5 confidence features
+ *   pos   [L, 16]  position embedding
+ *   W0    [S, 2r]  Init: u_0 = tanh(W0 [P_h h_ctx ; P_e E_in(x0)])
+ *   Wz,Wh [S, 2r+32] minimal-GRU gate and candidate over [P_h m_i ; P_e E_in(x_{i-1}) ; pos_i ; P_phi phi_i]
+ *   W_s   [r, S]   state side of the low-rank residual
+ *   W_c   [r, d]   candidate side of the low-rank residual
+ *   w_g   [S+5]    gate weights over [s_i ; phi_i]
+ *   b_g, alpha     gate bias and gate scale: gamma_i = sigmoid(alpha) sigmoid(w_g.[s_i;phi_i] + b_g) */
+typedef struct brisk_params {
+  const void *E_in, *E_out;
+  const void *P_h, *P_e, *P_phi, *pos;
+  const void *W0, *Wz, *Wh, *W_s, *W_c, *w_g;
+  float b_g, alpha;
+} brisk_params;
+
+/* Inputs and outputs of the fused tail. Output pointers marked "optional" may be NULL, in
+ * which case the values are kept in the workspace only. */
+typedef struct brisk_tail_io {
+  const void *logits_q;     /* [B, L, V] proposal logits l^q                              */
+  const void *logits_p;     /* [B, L, V] verifier logits                                  */
+  const void *hidden;       /* [B, L, d] MASK hidden states m_i                           */
+  const void *h_ctx;        /* [B, d]    context hidden state h_c                         */
+  const int32_t *x0;        /* [B]       anchor token, the token before the block         */
+  const float *u_sel;       /* [B, L] uniforms in [0,1) for sample Select (else unused)    */
+  const float *u_acc;       /* [B, L] acceptance uniforms (stochastic verify)             */
+  const float *u_res;       /* [B, L] residual-resampling uniforms (stochastic verify)    */
+  int32_t *cand_ids;        /* optional [B, L, K] candidate ids, best first               */
+  float *cand_logprob;      /* optional [B, L, K] log q_i of the candidates               */
+  float *lse_q;             /* optional [B, L]    log-partition of the proposal rows      */
+  int32_t *sel_tokens;      /* optional [B, L]    selected tokens x_i                     */
+  float *refined;           /* optional [B, L, K] refined scores                          */
+  int32_t *accepted_len;    /* [B]    accepted prefix length a, 0..L                      */
+  int32_t *out_tokens;      /* [B, L] x_0..x_{a-1}, then the correction at a (if a < L), then -1 */
+  int32_t *correction;      /* [B]    correction token, -1 when a == L                    */
+  int32_t *next_anchor;     /* optional [B] last committed token (anchor of the next block) */
+} brisk_tail_io;
+
+/* Optional timing hooks: cudaEvent_t handles (as void*) recorded on `stream` right before
+ * and right after the vocabulary-sweep kernel of brisk_decode_tail. NULL fields are skipped. */
+typedef struct brisk_events {
+  void *sweep_begin, *sweep_end;
+} brisk_events;
+
+/* Bytes of workspace the entry points need for `dims` (256-byte multiple). The same
+ * workspace serves every entry point for these dims. 0 if dims are invalid. */
+size_t brisk_workspace_bytes(const brisk_dims *dims);
+
+/* Bytes of the folded corrector tables for `dims` (256-byte multiple); 0 if invalid. */
+size_t brisk_tables_bytes(const brisk_dims *dims);
+
+/* Fold the frozen vocabulary rows into the corrector's weights, once per weight set
+ * (App. C.2: E_in, E_out and the backbone stay frozen, so P_e E_in(v), W_c E_out(v) and
+ * their products with the GRU and residual matrices are fixed per token). Fills `tables`
+ * (brisk_tables_bytes(dims) bytes). Must run before brisk_corrector_select /
+ * brisk_decode_tail with these params; `params` buffers may be freed afterwards. */
+brisk_status brisk_corrector_prepare(const brisk_dims *dims, const brisk_params *params,
+                                     void *tables, void *stream);
+
+/* Step 1 (Sec. 3.3 "C_i = TopK(q_i, K)"; App. C.2 ordered candidate set S_j): for every row
+ * (b, i) of logits_q [B, L, V]: lse_q = max + log sum exp(l - max) over all V, the K ids of
+ * largest logit ordered by (logit descending, id ascending) in cand_ids [B, L, K], and
+ * cand_logprob = l(id) - lse_q. */
+brisk_status brisk_topk_candidates(const brisk_dims *dims, const void *logits_q,
+                                   int32_t *cand_ids, float *cand_logprob, float *lse_q,
+                                   void *workspace, void *stream);
+
+/* Step 2 (Sec. 3.3 Eqs. 4-5; App. C.2 Eq. 7; Algorithm 1(b) loop): per sequence, sequentially
+ * over positions, the minimal-GRU corrector state, the gated low-rank residual on the K
+ * candidates and Select. Reads the step-1 outputs (cand_ids, cand_logprob) and logits_q
+ * (for the confidence features), hidden [B, L, d], h_ctx [B, d], x0 [B]; u_sel [B, L] is
+ * required for BRISK_SELECT_SAMPLE. Writes sel_tokens [B, L] and refined [B, L, K]
+ * (refined_{i,k} = cand_logprob_{i,k} + gamma_i d_{i,k}). `tables` from brisk_corrector_prepare. */
+brisk_status brisk_corrector_select(const brisk_dims *dims, const brisk_params *params,
+                                    const void *tables, const void *hidden, const void *h_ctx,
+                                    const int32_t *x0, const void *logits_q,
+                                    const int32_t *cand_ids, const float *cand_logprob,
+                                    int32_t select_mode, const float *u_sel,
+                                    int32_t *sel_tokens, float *refined,
+                                    void *workspace, void *stream);
+
+/* Step 3 (Sec. 3.1 accept-prefix; Sec. 3.3 speculative sampling; App. B Eq. 8 strict u < alpha):
+ * verifier row statistics over logits_p [B, L, V], then per sequence left to right to the first
+ * rejection. Greedy: accept iff sel_tokens[b,i] is the verifier argmax (lowest id on ties); the
+ * correction is that argmax. Stochastic: pi_i is softmax(refined) on cand_ids for sample Select and
+ * a point mass on the selected token for greedy Select; accept iff u_acc < min(1, p/pi); at the
+ * first rejection draw from the normalised [p - pi]_+ with u_res, walking ids in ascending order
+ * (the verifier argmax when that mass is <= 1e-6). Writes accepted_len [B], out_tokens [B, L] and
+ * correction [B]. */
+brisk_status brisk_verify_block(const brisk_dims *dims, const void *logits_p,
+                                const int32_t *sel_tokens, const int32_t *cand_ids,
+                                const float *refined, int32_t select_mode, int32_t verify_mode,
+                                const float *u_acc, const float *u_res, int32_t *accepted_len,
+                                int32_t *out_tokens, int32_t *correction, void *workspace,
+                                void *stream);
+
+/* Steps 1-3 for one block step (Algorithm 1(b) lines after the backbone pass): the same results,
+ * bit for bit, as brisk_topk_candidates + brisk_corrector_select + brisk_verify_block on the same
+ * inputs, with both logit tensors swept by one kernel. `ev` may be NULL. */
+brisk_status brisk_decode_tail(const brisk_dims *dims, const brisk_params *params,
+                               const void *tables, const brisk_tail_io *io, int32_t select_mode,
+                               int32_t verify_mode, void *workspace, const brisk_events *ev,
+                               void *stream);
+
+/* Kernels one brisk_decode_tail call launches for `dims` (0 if dims are invalid). */
+int32_t brisk_kernels_per_tail(const brisk_dims *dims);
+
+/* Reads the device status word of `workspace` (synchronises `stream`): BRISK_OK or the first
+ * device-side problem recorded by the most recent call on this workspace (every call clears the
+ * word when it starts). Device-side problems: a non-finite log-partition or a candidate id that
+ * a row with no finite logit left out of range (BRISK_ERR_NUMERIC); an anchor or selected token
+ * outside [0, V) (BRISK_ERR_INVALID_ARG; the id is replaced by 0 so that nothing reads out of
+ * bounds). With clear != 0 the word is reset to BRISK_OK afterwards. */
+brisk_status brisk_last_device_status(void *workspace, int32_t clear, void *stream);
+
+/* Human-readable name of a status code (static storage). */
+const char *brisk_status_string(brisk_status status);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* BRISK_H */

@@ -255,6 +255,7 @@ class VerifyResult:
     correction: int               # -1 when the whole block is accepted
     accept_margin: float = np.inf  # min |u_acc - alpha| over decided positions
     resample_margin: float = np.inf
+    accept_margins: Optional[np.ndarray] = None  # [L] |u_acc - alpha| per decided position
 
 
 def residual_sample(row_p: np.ndarray, pi_ids: Sequence[int], pi_mass: Sequence[float], u: float):
@@ -287,6 +288,7 @@ def verify_sequence(rows_p: Callable[[int], np.ndarray], sel_tokens: np.ndarray,
     L = len(sel_tokens)
     out = np.full(L, -1, dtype=np.int64)
     acc_margin = np.inf
+    margins = np.full(L, np.inf)
     for i in range(L):
         row = np.asarray(rows_p(i), dtype=np.float64)
         x = int(sel_tokens[i])
@@ -299,7 +301,8 @@ def verify_sequence(rows_p: Callable[[int], np.ndarray], sel_tokens: np.ndarray,
             p_x = np.exp(row[x] - log_partition(row))
             alpha = min(1.0, p_x / pi[rank])
             ok = float(u_acc[i]) < alpha
-            acc_margin = min(acc_margin, abs(float(u_acc[i]) - alpha))
+            margins[i] = abs(float(u_acc[i]) - alpha)
+            acc_margin = min(acc_margin, margins[i])
         if force_accept and i in force_accept:
             ok = bool(force_accept[i])
         if ok:
@@ -313,8 +316,8 @@ def verify_sequence(rows_p: Callable[[int], np.ndarray], sel_tokens: np.ndarray,
         if force_correction is not None:
             corr = int(force_correction)
         out[i] = corr
-        return VerifyResult(i, out, int(corr), acc_margin, res_margin)
-    return VerifyResult(L, out, -1, acc_margin, np.inf)
+        return VerifyResult(i, out, int(corr), acc_margin, res_margin, margins)
+    return VerifyResult(L, out, -1, acc_margin, np.inf, margins)
 
 
 # ---------------------------------------------------------------------------

@@ -4,14 +4,12 @@ The compute runs in the CUDA library built from ``csrc/``; ``brisk`` is its
 thin ctypes binding (loaded on first use). ``synth`` builds seeded synthetic
 inputs shaped like the paper's workloads.
 """
-__all__ = ["synth", "brisk"]
+import importlib
+
+__all__ = ["synth", "brisk", "build"]
 
 
 def __getattr__(name):
-    if name == "brisk":
-        from . import brisk as _b
-        return _b
-    if name == "synth":
-        from . import synth as _s
-        return _s
+    if name in __all__:
+        return importlib.import_module(f"{__name__}.{name}")
     raise AttributeError(name)

@@ -1,0 +1,246 @@
+"""ctypes binding of ``libbrisk.so`` (the C ABI in ``include/brisk.h``).
+
+Argument marshalling only: every step of the decode tail runs in the CUDA
+library. Tensors are torch CUDA tensors; their data pointers and the current
+torch stream are handed to the library. Loading fails loudly when the library
+has not been built; nothing here falls back to another implementation.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from dataclasses import dataclass
+from typing import Dict, Optional
+
+import torch
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(HERE, "libbrisk.so")
+
+OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_CUDA, ERR_TIMEOUT, ERR_NUMERIC = range(6)
+DT_F32, DT_BF16 = 0, 1
+SELECT_GREEDY, SELECT_SAMPLE = 0, 1
+VERIFY_GREEDY, VERIFY_STOCHASTIC = 0, 1
+
+_vp = ctypes.c_void_p
+
+
+class Dims(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_int32) for n in
+                ("B", "L", "V", "d", "K", "r", "logits_dtype", "hidden_dtype")]
+
+
+class Params(ctypes.Structure):
+    _fields_ = [(n, _vp) for n in ("E_in", "E_out", "P_h", "P_e", "P_phi", "pos", "W0", "Wz", "Wh",
+                                   "W_s", "W_c", "w_g")] + [("b_g", ctypes.c_float),
+                                                           ("alpha", ctypes.c_float)]
+
+
+class TailIO(ctypes.Structure):
+    _fields_ = [(n, _vp) for n in ("logits_q", "logits_p", "hidden", "h_ctx", "x0", "u_sel", "u_acc",
+                                   "u_res", "cand_ids", "cand_logprob", "lse_q", "sel_tokens",
+                                   "refined", "accepted_len", "out_tokens", "correction",
+                                   "next_anchor")]
+
+
+class Events(ctypes.Structure):
+    _fields_ = [("sweep_begin", _vp), ("sweep_end", _vp)]
+
+
+class BriskError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        super().__init__(f"{where}: {status_string(status)}")
+
+
+_lib = None
+
+# (name, restype, argtypes) of every exported entry point
+_SIGS = [
+    ("brisk_workspace_bytes", ctypes.c_size_t, [ctypes.POINTER(Dims)]),
+    ("brisk_tables_bytes", ctypes.c_size_t, [ctypes.POINTER(Dims)]),
+    ("brisk_corrector_prepare", ctypes.c_int, [ctypes.POINTER(Dims), ctypes.POINTER(Params), _vp, _vp]),
+    ("brisk_topk_candidates", ctypes.c_int, [ctypes.POINTER(Dims), _vp, _vp, _vp, _vp, _vp, _vp]),
+    ("brisk_corrector_select", ctypes.c_int,
+     [ctypes.POINTER(Dims), ctypes.POINTER(Params), _vp, _vp, _vp, _vp, _vp, _vp, _vp,
+      ctypes.c_int32, _vp, _vp, _vp, _vp, _vp]),
+    ("brisk_verify_block", ctypes.c_int,
+     [ctypes.POINTER(Dims), _vp, _vp, _vp, _vp, ctypes.c_int32, ctypes.c_int32, _vp, _vp, _vp, _vp,
+      _vp, _vp, _vp]),
+    ("brisk_decode_tail", ctypes.c_int,
+     [ctypes.POINTER(Dims), ctypes.POINTER(Params), _vp, ctypes.POINTER(TailIO), ctypes.c_int32,
+      ctypes.c_int32, _vp, ctypes.POINTER(Events), _vp]),
+    ("brisk_kernels_per_tail", ctypes.c_int32, [ctypes.POINTER(Dims)]),
+    ("brisk_last_device_status", ctypes.c_int, [_vp, ctypes.c_int32, _vp]),
+    ("brisk_status_string", ctypes.c_char_p, [ctypes.c_int]),
+]
+
+
+def lib():
+    """The loaded library; raises if it has not been built."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(f"{LIB_PATH} is missing: build it with "
+                               "`python -c 'import __graft_entry__ as g; g.build()'`")
+        h = ctypes.CDLL(LIB_PATH)
+        for name, res, args in _SIGS:
+            f = getattr(h, name)
+            f.restype = res
+            f.argtypes = args
+        _lib = h
+    return _lib
+
+
+def status_string(s: int) -> str:
+    return lib().brisk_status_string(int(s)).decode()
+
+
+def _check(s: int, where: str) -> None:
+    if s != OK:
+        raise BriskError(s, where)
+
+
+def _dt(t: torch.dtype) -> int:
+    if t == torch.bfloat16:
+        return DT_BF16
+    if t == torch.float32:
+        return DT_F32
+    raise ValueError(f"unsupported dtype {t}")
+
+
+def _p(t: Optional[torch.Tensor]):
+    if t is None:
+        return None
+    if not t.is_contiguous():
+        raise ValueError("tensors must be contiguous")
+    return _vp(t.data_ptr())
+
+
+def _stream(stream=None):
+    s = torch.cuda.current_stream() if stream is None else stream
+    return _vp(s.cuda_stream)
+
+
+def make_dims(B, L, V, d, K, r, logits_dtype, hidden_dtype) -> Dims:
+    return Dims(B, L, V, d, K, r, _dt(logits_dtype), _dt(hidden_dtype))
+
+
+def workspace_bytes(dims: Dims) -> int:
+    return int(lib().brisk_workspace_bytes(ctypes.byref(dims)))
+
+
+def tables_bytes(dims: Dims) -> int:
+    return int(lib().brisk_tables_bytes(ctypes.byref(dims)))
+
+
+def kernels_per_tail(dims: Dims) -> int:
+    return int(lib().brisk_kernels_per_tail(ctypes.byref(dims)))
+
+
+def make_params(w: Dict[str, object]) -> Params:
+    names = ("E_in", "E_out", "P_h", "P_e", "P_phi", "pos", "W0", "Wz", "Wh", "W_s", "W_c", "w_g")
+    return Params(*[_p(w[n]) for n in names], float(w["b_g"]), float(w["alpha"]))
+
+
+class DecodeTail:
+    """Device buffers and calls of the decode tail for one problem size and weight set.
+
+    ``weights`` holds the corrector parameters and E_in / E_out as CUDA tensors in the hidden
+    dtype (see ``synth.make_weights``). The workspace and the folded tables are allocated once
+    here with torch; the library itself never allocates.
+    """
+
+    def __init__(self, B, L, V, d, K, r, logits_dtype, hidden_dtype, weights, device="cuda"):
+        self.dims = make_dims(B, L, V, d, K, r, logits_dtype, hidden_dtype)
+        self.B, self.L, self.V, self.d, self.K, self.r = B, L, V, d, K, r
+        self.device = torch.device(device)
+        ws = workspace_bytes(self.dims)
+        tb = tables_bytes(self.dims)
+        if ws == 0 or tb == 0:
+            raise BriskError(ERR_INVALID_ARG, "dims")
+        self.workspace = torch.zeros(ws, dtype=torch.uint8, device=self.device)
+        self.tables = torch.empty(tb, dtype=torch.uint8, device=self.device)
+        self.weights = weights
+        self.params = make_params(weights)
+        self.prepared = False
+
+    @classmethod
+    def for_workload(cls, wl, weights, device="cuda", B=None):
+        return cls(wl.B if B is None else B, wl.L, wl.V, wl.d, wl.K, wl.r, wl.logits_dtype,
+                   wl.hidden_dtype, weights, device)
+
+    def prepare(self, stream=None):
+        _check(lib().brisk_corrector_prepare(ctypes.byref(self.dims), ctypes.byref(self.params),
+                                             _p(self.tables), _stream(stream)), "prepare")
+        self.prepared = True
+
+    def _i32(self, *shape):
+        return torch.empty(shape, dtype=torch.int32, device=self.device)
+
+    def _f32(self, *shape):
+        return torch.empty(shape, dtype=torch.float32, device=self.device)
+
+    def topk(self, logits_q, stream=None):
+        B, L, K = self.B, self.L, self.K
+        ids, lp, lse = self._i32(B, L, K), self._f32(B, L, K), self._f32(B, L)
+        _check(lib().brisk_topk_candidates(ctypes.byref(self.dims), _p(logits_q), _p(ids), _p(lp),
+                                           _p(lse), _p(self.workspace), _stream(stream)), "topk")
+        return {"cand_ids": ids, "cand_logprob": lp, "lse_q": lse}
+
+    def select(self, hidden, h_ctx, x0, logits_q, cand_ids, cand_logprob, select_mode=SELECT_GREEDY,
+               u_sel=None, stream=None):
+        B, L, K = self.B, self.L, self.K
+        sel, ref = self._i32(B, L), self._f32(B, L, K)
+        _check(lib().brisk_corrector_select(
+            ctypes.byref(self.dims), ctypes.byref(self.params), _p(self.tables), _p(hidden), _p(h_ctx),
+            _p(x0), _p(logits_q), _p(cand_ids), _p(cand_logprob), int(select_mode), _p(u_sel),
+            _p(sel), _p(ref), _p(self.workspace), _stream(stream)), "select")
+        return {"sel_tokens": sel, "refined": ref}
+
+    def verify(self, logits_p, sel_tokens, cand_ids, refined, select_mode=SELECT_GREEDY,
+               verify_mode=VERIFY_GREEDY, u_acc=None, u_res=None, stream=None):
+        B, L = self.B, self.L
+        a, out, corr = self._i32(B), self._i32(B, L), self._i32(B)
+        _check(lib().brisk_verify_block(
+            ctypes.byref(self.dims), _p(logits_p), _p(sel_tokens), _p(cand_ids), _p(refined),
+            int(select_mode), int(verify_mode), _p(u_acc), _p(u_res), _p(a), _p(out), _p(corr),
+            _p(self.workspace), _stream(stream)), "verify")
+        return {"accepted_len": a, "out_tokens": out, "correction": corr}
+
+    def alloc_outputs(self, full=True):
+        B, L, K = self.B, self.L, self.K
+        o = {"accepted_len": self._i32(B), "out_tokens": self._i32(B, L), "correction": self._i32(B),
+             "next_anchor": self._i32(B)}
+        if full:
+            o.update(cand_ids=self._i32(B, L, K), cand_logprob=self._f32(B, L, K),
+                     lse_q=self._f32(B, L), sel_tokens=self._i32(B, L), refined=self._f32(B, L, K))
+        return o
+
+    def tail(self, block, select_mode=SELECT_GREEDY, verify_mode=VERIFY_GREEDY, out=None, x0=None,
+             events=None, stream=None):
+        """One fused decode-tail call on the tensors of ``block`` (see ``synth.make_block``)."""
+        if out is None:
+            out = self.alloc_outputs()
+        io = TailIO(_p(block["logits_q"]), _p(block["logits_p"]), _p(block["hidden"]),
+                    _p(block["h_c"]), _p(block["x0"] if x0 is None else x0), _p(block.get("u_sel")),
+                    _p(block.get("u_acc")), _p(block.get("u_res")), _p(out.get("cand_ids")),
+                    _p(out.get("cand_logprob")), _p(out.get("lse_q")), _p(out.get("sel_tokens")),
+                    _p(out.get("refined")), _p(out["accepted_len"]), _p(out["out_tokens"]),
+                    _p(out["correction"]), _p(out.get("next_anchor")))
+        ev = None
+        if events is not None:
+            ev = ctypes.byref(Events(_vp(events[0].cuda_event), _vp(events[1].cuda_event)))
+        _check(lib().brisk_decode_tail(ctypes.byref(self.dims), ctypes.byref(self.params),
+                                       _p(self.tables), ctypes.byref(io), int(select_mode),
+                                       int(verify_mode), _p(self.workspace), ev, _stream(stream)),
+               "decode_tail")
+        return out
+
+    def device_status(self, clear=True, stream=None) -> int:
+        return int(lib().brisk_last_device_status(_p(self.workspace), int(clear), _stream(stream)))
+
+
+def mode_ids(select_mode: str, verify_mode: str):
+    return (SELECT_SAMPLE if select_mode == "sample" else SELECT_GREEDY,
+            VERIFY_STOCHASTIC if verify_mode == "stochastic" else VERIFY_GREEDY)

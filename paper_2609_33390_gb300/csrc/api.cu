@@ -1,0 +1,440 @@
+// C ABI of the decode tail: argument checks, workspace and table layouts, launches.
+#include <string.h>
+
+#include "brisk_internal.cuh"
+
+using namespace brisk;
+
+namespace {
+
+constexpr size_t ALIGN = 256;
+inline size_t up(size_t x) { return (x + ALIGN - 1) / ALIGN * ALIGN; }
+
+bool dims_ok(const brisk_dims* d) {
+  if (!d) return false;
+  if (d->B < 1 || d->L < 1 || d->L > 64) return false;
+  if (d->K < 4 || d->K > 32 || d->V < d->K) return false;
+  if (d->d < 8 || d->d % 8 != 0) return false;
+  if (d->r < 16 || d->r > 512 || d->r % 16 != 0) return false;
+  if ((d->logits_dtype != BRISK_DT_F32 && d->logits_dtype != BRISK_DT_BF16) ||
+      (d->hidden_dtype != BRISK_DT_F32 && d->hidden_dtype != BRISK_DT_BF16))
+    return false;
+  if ((long long)d->B * d->L * d->V > (1LL << 40)) return false;
+  return true;
+}
+
+inline size_t esize(int dt) { return dt == BRISK_DT_BF16 ? 2 : 4; }
+
+// ---------------------------------------------------------------- workspace layout
+struct WsLayout {
+  size_t status, counters, part_val, part_id, part_m, part_s, argmax_p, lse_p;
+  size_t cand_ids, cand_logprob, lse_q, sel, refined, Hm, G, G0, total;
+  int nchunk, KP;
+};
+
+WsLayout ws_layout(const brisk_dims* d) {
+  WsLayout w{};
+  const size_t BL = (size_t)d->B * d->L;
+  const size_t S = 2 * (size_t)d->r;
+  w.nchunk = sweep_chunks((int)BL, d->V, d->logits_dtype, 0);
+  w.KP = kp_for(d->K);
+  const size_t np = 2 * BL * w.nchunk;
+  size_t o = 0;
+  auto take = [&](size_t bytes) { const size_t r = o; o = up(o + bytes); return r; };
+  w.status = take(ALIGN);
+  w.counters = take(sizeof(int32_t) * 2 * BL);
+  w.part_val = take(sizeof(float) * np * w.KP);
+  w.part_id = take(sizeof(int32_t) * np * w.KP);
+  w.part_m = take(sizeof(float) * np);
+  w.part_s = take(sizeof(float) * np);
+  w.argmax_p = take(sizeof(int32_t) * BL);
+  w.lse_p = take(sizeof(float) * BL);
+  w.cand_ids = take(sizeof(int32_t) * BL * d->K);
+  w.cand_logprob = take(sizeof(float) * BL * d->K);
+  w.lse_q = take(sizeof(float) * BL);
+  w.sel = take(sizeof(int32_t) * BL);
+  w.refined = take(sizeof(float) * BL * d->K);
+  w.Hm = take(sizeof(float) * (BL + d->B) * d->r);
+  w.G = take(sizeof(float) * BL * 2 * S);
+  w.G0 = take(sizeof(float) * d->B * S);
+  w.total = o;
+  return w;
+}
+
+// ---------------------------------------------------------------- folded tables layout
+// Tzh [V, 2S]: token share of the GRU pre-activations, Tz(v) | Th(v) with
+//              Tz(v) = W_z[:, r:2r] P_e E_in(v), Th(v) = W_h[:, r:2r] P_e E_in(v)
+// U   [V, S] : residual rows, U(v) = W_s^T W_c E_out(v)
+// T0  [V, S] : token share of Init, W0[:, r:2r] P_e E_in(v)
+// Tin, Tout [V, r]: P_e E_in(v), W_c E_out(v) (intermediates of the folds)
+// posz, posh [L, S]: position shares W_z[:, 2r:2r+16] pos_i, W_h[:, 2r:2r+16] pos_i
+// Fz, Fh [S, 5]: feature shares W_z[:, 2r+16:] P_phi, W_h[:, 2r+16:] P_phi
+// wg [S+5] fp32 copy of w_g; W2 [2S, r] = [W_z[:, :r] ; W_h[:, :r]] and W0h [S, r] = W0[:, :r] (fp32)
+struct TbLayout {
+  size_t Tzh, U, T0, Tin, Tout, posz, posh, Fz, Fh, wg, W2, W0h, total;
+};
+
+TbLayout tb_layout(const brisk_dims* d) {
+  TbLayout t{};
+  const size_t V = d->V, r = d->r, S = 2 * r, L = d->L;
+  size_t o = 0;
+  auto take = [&](size_t bytes) { const size_t q = o; o = up(o + bytes); return q; };
+  t.Tzh = take(sizeof(float) * V * 2 * S);
+  t.U = take(sizeof(float) * V * S);
+  t.T0 = take(sizeof(float) * V * S);
+  t.Tin = take(sizeof(float) * V * r);
+  t.Tout = take(sizeof(float) * V * r);
+  t.posz = take(sizeof(float) * L * S);
+  t.posh = take(sizeof(float) * L * S);
+  t.Fz = take(sizeof(float) * S * 5);
+  t.Fh = take(sizeof(float) * S * 5);
+  t.wg = take(sizeof(float) * (S + 5));
+  t.W2 = take(sizeof(float) * 2 * S * r);
+  t.W0h = take(sizeof(float) * S * r);
+  t.total = o;
+  return t;
+}
+
+template <typename T>
+inline T* at(void* base, size_t off) { return reinterpret_cast<T*>(static_cast<char*>(base) + off); }
+template <typename T>
+inline const T* at(const void* base, size_t off) {
+  return reinterpret_cast<const T*>(static_cast<const char*>(base) + off);
+}
+
+inline bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+#define BRISK_CUDA(call)                       \
+  do {                                         \
+    if ((call) != cudaSuccess) return BRISK_ERR_CUDA; \
+  } while (0)
+
+bool params_ok(const brisk_params* p) {
+  return p && p->E_in && p->E_out && p->P_h && p->P_e && p->P_phi && p->pos && p->W0 && p->Wz &&
+         p->Wh && p->W_s && p->W_c && p->w_g;
+}
+
+// Clears the status word and the sweep arrival counters of a workspace.
+brisk_status clear_ws(const WsLayout& w, const brisk_dims* d, void* ws, cudaStream_t st) {
+  BRISK_CUDA(cudaMemsetAsync(ws, 0, w.counters + sizeof(int32_t) * 2 * (size_t)d->B * d->L, st));
+  return BRISK_OK;
+}
+
+SweepSeg make_seg(const WsLayout& w, void* ws, int seg, const void* logits, int rows, int kout,
+                  int32_t* out_ids, float* out_logprob, float* out_lse) {
+  SweepSeg s{};
+  const size_t np = (size_t)rows * w.nchunk;
+  const size_t off = seg * np;
+  s.logits = logits;
+  s.rows = rows;
+  s.kout = kout;
+  s.out_ids = out_ids;
+  s.out_logprob = out_logprob;
+  s.out_lse = out_lse;
+  s.part_val = at<float>(ws, w.part_val) + off * w.KP;
+  s.part_id = at<int32_t>(ws, w.part_id) + off * w.KP;
+  s.part_m = at<float>(ws, w.part_m) + off;
+  s.part_s = at<float>(ws, w.part_s) + off;
+  s.counters = at<int32_t>(ws, w.counters) + (size_t)seg * rows;
+  return s;
+}
+
+// The hidden-state shares of the corrector: Hm = [hidden ; h_ctx] P_h^T, then
+// G = Hm[:BL] [W_z[:, :r] ; W_h[:, :r]]^T and G0 = Hm[BL:] W0[:, :r]^T.
+brisk_status hidden_products(const brisk_dims* d, const brisk_params* p, const void* tables,
+                             const void* hidden, const void* h_ctx, const WsLayout& w, void* ws,
+                             cudaStream_t st) {
+  const TbLayout t = tb_layout(d);
+  const int BL = d->B * d->L, r = d->r, S = 2 * d->r, hd = d->hidden_dtype;
+  float* Hm = at<float>(ws, w.Hm);
+  BRISK_CUDA(gemm_simt(BL, r, d->d, hidden, hd, d->d, p->P_h, hd, d->d, false, Hm, r, st));
+  BRISK_CUDA(gemm_simt(d->B, r, d->d, h_ctx, hd, d->d, p->P_h, hd, d->d, false,
+                       Hm + (size_t)BL * r, r, st));
+  BRISK_CUDA(gemm_simt(BL, 2 * S, r, Hm, BRISK_DT_F32, r, at<float>(tables, t.W2), BRISK_DT_F32, r,
+                       false, at<float>(ws, w.G), 2 * S, st));
+  BRISK_CUDA(gemm_simt(d->B, S, r, Hm + (size_t)BL * r, BRISK_DT_F32, r, at<float>(tables, t.W0h),
+                       BRISK_DT_F32, r, false, at<float>(ws, w.G0), S, st));
+  return BRISK_OK;
+}
+
+ScanArgs scan_args(const brisk_dims* d, const brisk_params* p, const void* tables, const WsLayout& w,
+                   void* ws) {
+  ScanArgs a{};
+  a.B = d->B; a.L = d->L; a.V = d->V; a.K = d->K; a.S = 2 * d->r; a.logits_dt = d->logits_dtype;
+  a.status = at<int32_t>(ws, w.status);
+  if (tables) {
+    const TbLayout t = tb_layout(d);
+    a.Tzh = at<float>(tables, t.Tzh);
+    a.U = at<float>(tables, t.U);
+    a.T0 = at<float>(tables, t.T0);
+    a.posz = at<float>(tables, t.posz);
+    a.posh = at<float>(tables, t.posh);
+    a.Fz = at<float>(tables, t.Fz);
+    a.Fh = at<float>(tables, t.Fh);
+    a.wg = at<float>(tables, t.wg);
+  }
+  if (p) {
+    a.b_g = p->b_g;
+    a.alpha = p->alpha;
+  }
+  a.G = at<float>(ws, w.G);
+  a.G0 = at<float>(ws, w.G0);
+  a.argmax_p = at<int32_t>(ws, w.argmax_p);
+  a.lse_p = at<float>(ws, w.lse_p);
+  return a;
+}
+
+}  // namespace
+
+extern "C" {
+
+size_t brisk_workspace_bytes(const brisk_dims* dims) {
+  if (!dims_ok(dims)) return 0;
+  return ws_layout(dims).total;
+}
+
+size_t brisk_tables_bytes(const brisk_dims* dims) {
+  if (!dims_ok(dims)) return 0;
+  return tb_layout(dims).total;
+}
+
+const char* brisk_status_string(brisk_status s) {
+  switch (s) {
+    case BRISK_OK: return "BRISK_OK";
+    case BRISK_ERR_INVALID_ARG: return "BRISK_ERR_INVALID_ARG";
+    case BRISK_ERR_UNSUPPORTED: return "BRISK_ERR_UNSUPPORTED";
+    case BRISK_ERR_CUDA: return "BRISK_ERR_CUDA";
+    case BRISK_ERR_TIMEOUT: return "BRISK_ERR_TIMEOUT";
+    case BRISK_ERR_NUMERIC: return "BRISK_ERR_NUMERIC";
+  }
+  return "BRISK_ERR_UNKNOWN";
+}
+
+brisk_status brisk_corrector_prepare(const brisk_dims* d, const brisk_params* p, void* tables,
+                                     void* stream) {
+  if (!dims_ok(d) || !params_ok(p) || !tables || !aligned(tables, ALIGN)) return BRISK_ERR_INVALID_ARG;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const TbLayout t = tb_layout(d);
+  const int V = d->V, r = d->r, S = 2 * r, L = d->L, hd = d->hidden_dtype, F32 = BRISK_DT_F32;
+  const int ldw = 2 * r + 32;
+  const size_t es = esize(hd);
+  auto wp = [&](const void* base, size_t elems) {
+    return static_cast<const void*>(static_cast<const char*>(base) + elems * es);
+  };
+  float* Tin = at<float>(tables, t.Tin);
+  float* Tout = at<float>(tables, t.Tout);
+  float* Tzh = at<float>(tables, t.Tzh);
+  // P_e E_in(v) and W_c E_out(v) for every v
+  BRISK_CUDA(gemm_simt(V, r, d->d, p->E_in, hd, d->d, p->P_e, hd, d->d, false, Tin, r, st));
+  BRISK_CUDA(gemm_simt(V, r, d->d, p->E_out, hd, d->d, p->W_c, hd, d->d, false, Tout, r, st));
+  // token shares of the gate / candidate pre-activations and of Init
+  BRISK_CUDA(gemm_simt(V, S, r, Tin, F32, r, wp(p->Wz, r), hd, ldw, false, Tzh, 2 * S, st));
+  BRISK_CUDA(gemm_simt(V, S, r, Tin, F32, r, wp(p->Wh, r), hd, ldw, false, Tzh + S, 2 * S, st));
+  BRISK_CUDA(gemm_simt(V, S, r, Tin, F32, r, wp(p->W0, r), hd, 2 * r, false, at<float>(tables, t.T0),
+                       S, st));
+  // residual rows U(v) = W_s^T (W_c E_out(v)): B(n=j, k=t) = W_s[t, j]
+  BRISK_CUDA(gemm_simt(V, S, r, Tout, F32, r, p->W_s, hd, S, true, at<float>(tables, t.U), S, st));
+  // position shares
+  BRISK_CUDA(gemm_simt(L, S, 16, p->pos, hd, 16, wp(p->Wz, 2 * r), hd, ldw, false,
+                       at<float>(tables, t.posz), S, st));
+  BRISK_CUDA(gemm_simt(L, S, 16, p->pos, hd, 16, wp(p->Wh, 2 * r), hd, ldw, false,
+                       at<float>(tables, t.posh), S, st));
+  // feature shares: F(j, f) = sum_t W[j, 2r+16+t] P_phi[t, f]
+  BRISK_CUDA(gemm_simt(S, 5, 16, wp(p->Wz, 2 * r + 16), hd, ldw, p->P_phi, hd, 5, true,
+                       at<float>(tables, t.Fz), 5, st));
+  BRISK_CUDA(gemm_simt(S, 5, 16, wp(p->Wh, 2 * r + 16), hd, ldw, p->P_phi, hd, 5, true,
+                       at<float>(tables, t.Fh), 5, st));
+  // fp32 copies of the gate weights and of the hidden-state blocks
+  BRISK_CUDA(copy2d(1, S + 5, p->w_g, hd, S + 5, at<float>(tables, t.wg), F32, S + 5, st));
+  BRISK_CUDA(copy2d(S, r, p->Wz, hd, ldw, at<float>(tables, t.W2), F32, r, st));
+  BRISK_CUDA(copy2d(S, r, p->Wh, hd, ldw, at<float>(tables, t.W2) + (size_t)S * r, F32, r, st));
+  BRISK_CUDA(copy2d(S, r, p->W0, hd, 2 * r, at<float>(tables, t.W0h), F32, r, st));
+  return BRISK_OK;
+}
+
+brisk_status brisk_topk_candidates(const brisk_dims* d, const void* logits_q, int32_t* cand_ids,
+                                   float* cand_logprob, float* lse_q, void* ws, void* stream) {
+  if (!dims_ok(d) || !logits_q || !cand_ids || !cand_logprob || !lse_q || !ws ||
+      !aligned(ws, ALIGN) || !aligned(logits_q, esize(d->logits_dtype)))
+    return BRISK_ERR_INVALID_ARG;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const WsLayout w = ws_layout(d);
+  brisk_status s = clear_ws(w, d, ws, st);
+  if (s != BRISK_OK) return s;
+  SweepLaunch a{};
+  a.seg[0] = make_seg(w, ws, 0, logits_q, d->B * d->L, d->K, cand_ids, cand_logprob, lse_q);
+  a.nseg = 1;
+  a.V = d->V;
+  a.nchunk = w.nchunk;
+  a.KP = w.KP;
+  a.dtype = d->logits_dtype;
+  a.status = at<int32_t>(ws, w.status);
+  BRISK_CUDA(launch_sweep(a, st));
+  return BRISK_OK;
+}
+
+brisk_status brisk_corrector_select(const brisk_dims* d, const brisk_params* p, const void* tables,
+                                    const void* hidden, const void* h_ctx, const int32_t* x0,
+                                    const void* logits_q, const int32_t* cand_ids,
+                                    const float* cand_logprob, int32_t select_mode,
+                                    const float* u_sel, int32_t* sel_tokens, float* refined,
+                                    void* ws, void* stream) {
+  if (!dims_ok(d) || !params_ok(p) || !tables || !hidden || !h_ctx || !x0 || !logits_q ||
+      !cand_ids || !cand_logprob || !sel_tokens || !refined || !ws || !aligned(ws, ALIGN) ||
+      !aligned(tables, ALIGN))
+    return BRISK_ERR_INVALID_ARG;
+  if (select_mode != BRISK_SELECT_GREEDY && select_mode != BRISK_SELECT_SAMPLE)
+    return BRISK_ERR_INVALID_ARG;
+  if (select_mode == BRISK_SELECT_SAMPLE && !u_sel) return BRISK_ERR_INVALID_ARG;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const WsLayout w = ws_layout(d);
+  brisk_status s = clear_ws(w, d, ws, st);
+  if (s != BRISK_OK) return s;
+  s = hidden_products(d, p, tables, hidden, h_ctx, w, ws, st);
+  if (s != BRISK_OK) return s;
+  ScanArgs a = scan_args(d, p, tables, w, ws);
+  a.select_mode = select_mode;
+  a.do_select = 1;
+  a.do_verify = 0;
+  a.logits_q = logits_q;
+  a.cand_ids = cand_ids;
+  a.cand_logprob = cand_logprob;
+  a.x0 = x0;
+  a.u_sel = u_sel;
+  a.sel_tokens = sel_tokens;
+  a.refined = refined;
+  BRISK_CUDA(launch_scan(a, st));
+  return BRISK_OK;
+}
+
+brisk_status brisk_verify_block(const brisk_dims* d, const void* logits_p, const int32_t* sel_tokens,
+                                const int32_t* cand_ids, const float* refined, int32_t select_mode,
+                                int32_t verify_mode, const float* u_acc, const float* u_res,
+                                int32_t* accepted_len, int32_t* out_tokens, int32_t* correction,
+                                void* ws, void* stream) {
+  if (!dims_ok(d) || !logits_p || !sel_tokens || !cand_ids || !refined || !accepted_len ||
+      !out_tokens || !correction || !ws || !aligned(ws, ALIGN) ||
+      !aligned(logits_p, esize(d->logits_dtype)))
+    return BRISK_ERR_INVALID_ARG;
+  if ((select_mode != BRISK_SELECT_GREEDY && select_mode != BRISK_SELECT_SAMPLE) ||
+      (verify_mode != BRISK_VERIFY_GREEDY && verify_mode != BRISK_VERIFY_STOCHASTIC))
+    return BRISK_ERR_INVALID_ARG;
+  if (verify_mode == BRISK_VERIFY_STOCHASTIC && (!u_acc || !u_res)) return BRISK_ERR_INVALID_ARG;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const WsLayout w = ws_layout(d);
+  brisk_status s = clear_ws(w, d, ws, st);
+  if (s != BRISK_OK) return s;
+  SweepLaunch sw{};
+  const int BL = d->B * d->L;
+  sw.seg[0] = make_seg(w, ws, 1, logits_p, BL, 1, at<int32_t>(ws, w.argmax_p), nullptr,
+                       at<float>(ws, w.lse_p));
+  sw.nseg = 1;
+  sw.V = d->V;
+  sw.nchunk = w.nchunk;
+  sw.KP = w.KP;
+  sw.dtype = d->logits_dtype;
+  sw.status = at<int32_t>(ws, w.status);
+  BRISK_CUDA(launch_sweep(sw, st));
+  ScanArgs a = scan_args(d, nullptr, nullptr, w, ws);
+  a.select_mode = select_mode;
+  a.verify_mode = verify_mode;
+  a.do_select = 0;
+  a.do_verify = 1;
+  a.cand_ids = cand_ids;
+  a.sel_tokens = const_cast<int32_t*>(sel_tokens);
+  a.refined = const_cast<float*>(refined);
+  a.logits_p = logits_p;
+  a.u_acc = u_acc;
+  a.u_res = u_res;
+  a.accepted_len = accepted_len;
+  a.out_tokens = out_tokens;
+  a.correction = correction;
+  BRISK_CUDA(launch_scan(a, st));
+  return BRISK_OK;
+}
+
+brisk_status brisk_decode_tail(const brisk_dims* d, const brisk_params* p, const void* tables,
+                               const brisk_tail_io* io, int32_t select_mode, int32_t verify_mode,
+                               void* ws, const brisk_events* ev, void* stream) {
+  if (!dims_ok(d) || !params_ok(p) || !tables || !io || !ws || !aligned(ws, ALIGN) ||
+      !aligned(tables, ALIGN))
+    return BRISK_ERR_INVALID_ARG;
+  if (!io->logits_q || !io->logits_p || !io->hidden || !io->h_ctx || !io->x0 || !io->accepted_len ||
+      !io->out_tokens || !io->correction)
+    return BRISK_ERR_INVALID_ARG;
+  if (!aligned(io->logits_q, esize(d->logits_dtype)) || !aligned(io->logits_p, esize(d->logits_dtype)))
+    return BRISK_ERR_INVALID_ARG;
+  if ((select_mode != BRISK_SELECT_GREEDY && select_mode != BRISK_SELECT_SAMPLE) ||
+      (verify_mode != BRISK_VERIFY_GREEDY && verify_mode != BRISK_VERIFY_STOCHASTIC))
+    return BRISK_ERR_INVALID_ARG;
+  if (select_mode == BRISK_SELECT_SAMPLE && !io->u_sel) return BRISK_ERR_INVALID_ARG;
+  if (verify_mode == BRISK_VERIFY_STOCHASTIC && (!io->u_acc || !io->u_res)) return BRISK_ERR_INVALID_ARG;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const WsLayout w = ws_layout(d);
+  brisk_status s = clear_ws(w, d, ws, st);
+  if (s != BRISK_OK) return s;
+  const int BL = d->B * d->L;
+  int32_t* cand_ids = io->cand_ids ? io->cand_ids : at<int32_t>(ws, w.cand_ids);
+  float* cand_lp = io->cand_logprob ? io->cand_logprob : at<float>(ws, w.cand_logprob);
+  float* lse_q = io->lse_q ? io->lse_q : at<float>(ws, w.lse_q);
+  int32_t* sel = io->sel_tokens ? io->sel_tokens : at<int32_t>(ws, w.sel);
+  float* refined = io->refined ? io->refined : at<float>(ws, w.refined);
+
+  SweepLaunch sw{};
+  sw.seg[0] = make_seg(w, ws, 0, io->logits_q, BL, d->K, cand_ids, cand_lp, lse_q);
+  sw.seg[1] = make_seg(w, ws, 1, io->logits_p, BL, 1, at<int32_t>(ws, w.argmax_p), nullptr,
+                       at<float>(ws, w.lse_p));
+  sw.nseg = 2;
+  sw.V = d->V;
+  sw.nchunk = w.nchunk;
+  sw.KP = w.KP;
+  sw.dtype = d->logits_dtype;
+  sw.status = at<int32_t>(ws, w.status);
+  if (ev && ev->sweep_begin) BRISK_CUDA(cudaEventRecord(static_cast<cudaEvent_t>(ev->sweep_begin), st));
+  BRISK_CUDA(launch_sweep(sw, st));
+  if (ev && ev->sweep_end) BRISK_CUDA(cudaEventRecord(static_cast<cudaEvent_t>(ev->sweep_end), st));
+
+  s = hidden_products(d, p, tables, io->hidden, io->h_ctx, w, ws, st);
+  if (s != BRISK_OK) return s;
+  ScanArgs a = scan_args(d, p, tables, w, ws);
+  a.select_mode = select_mode;
+  a.verify_mode = verify_mode;
+  a.do_select = 1;
+  a.do_verify = 1;
+  a.logits_q = io->logits_q;
+  a.cand_ids = cand_ids;
+  a.cand_logprob = cand_lp;
+  a.x0 = io->x0;
+  a.u_sel = io->u_sel;
+  a.sel_tokens = sel;
+  a.refined = refined;
+  a.logits_p = io->logits_p;
+  a.u_acc = io->u_acc;
+  a.u_res = io->u_res;
+  a.accepted_len = io->accepted_len;
+  a.out_tokens = io->out_tokens;
+  a.correction = io->correction;
+  a.next_anchor = io->next_anchor;
+  BRISK_CUDA(launch_scan(a, st));
+  return BRISK_OK;
+}
+
+int32_t brisk_kernels_per_tail(const brisk_dims* dims) {
+  if (!dims_ok(dims)) return 0;
+  return 1 /* sweep */ + 4 /* hidden-state products */ + 1 /* scan + verify */;
+}
+
+brisk_status brisk_last_device_status(void* ws, int32_t clear, void* stream) {
+  if (!ws) return BRISK_ERR_INVALID_ARG;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  int32_t h = 0;
+  BRISK_CUDA(cudaMemcpyAsync(&h, ws, sizeof(int32_t), cudaMemcpyDeviceToHost, st));
+  BRISK_CUDA(cudaStreamSynchronize(st));
+  if (clear) {
+    BRISK_CUDA(cudaMemsetAsync(ws, 0, sizeof(int32_t), st));
+    BRISK_CUDA(cudaStreamSynchronize(st));
+  }
+  return static_cast<brisk_status>(h);
+}
+
+}  // extern "C"

@@ -1,0 +1,228 @@
+// Internal declarations shared by the CUDA translation units of the decode tail.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <stdint.h>
+#include <math.h>
+
+#include "../../include/brisk.h"
+
+namespace brisk {
+
+constexpr unsigned FULL_MASK = 0xffffffffu;
+constexpr float LOG2E = 1.4426950408889634f;   // log2(e): exp(x) = 2^(x log2 e)
+constexpr float LN2 = 0.6931471805599453f;
+constexpr int INVALID_ID = 0x7fffffff;
+constexpr float RESID_Z_FLOOR = 1e-6f;         // residual mass below which the verifier argmax is used
+
+// ---------------------------------------------------------------- element access
+__device__ __forceinline__ float to_f32(float x) { return x; }
+__device__ __forceinline__ float to_f32(__nv_bfloat16 x) { return __bfloat162float(x); }
+
+template <typename T> struct Vec;   // 16-byte vector of T
+template <> struct Vec<float> { static constexpr int N = 4; };
+template <> struct Vec<__nv_bfloat16> { static constexpr int N = 8; };
+
+// Streaming 16-byte load that skips L1 allocation (each logit is read once).
+__device__ __forceinline__ uint4 ld_stream_v4(const void* p) {
+  uint4 r;
+  asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w) : "l"(p));
+  return r;
+}
+
+__device__ __forceinline__ void unpack(const uint4& w, float (&f)[8], __nv_bfloat16) {
+  const uint32_t u[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    f[2 * j] = __uint_as_float(u[j] << 16);
+    f[2 * j + 1] = __uint_as_float(u[j] & 0xffff0000u);
+  }
+}
+__device__ __forceinline__ void unpack(const uint4& w, float (&f)[4], float) {
+  f[0] = __uint_as_float(w.x);
+  f[1] = __uint_as_float(w.y);
+  f[2] = __uint_as_float(w.z);
+  f[3] = __uint_as_float(w.w);
+}
+
+// Hardware base-2 exponential (MUFU), flushes subnormal results to zero.
+__device__ __forceinline__ float ex2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+// ---------------------------------------------------------------- ordering
+// Candidate order of the method: logit descending, then id ascending.
+__device__ __forceinline__ bool better(float v1, int i1, float v2, int i2) {
+  return v1 > v2 || (v1 == v2 && i1 < i2);
+}
+
+// Insert (v, id) into a list sorted best-first; the worst entry falls off.
+template <int KP>
+__device__ __forceinline__ void list_insert(float v, int id, float (&vals)[KP], int (&ids)[KP]) {
+#pragma unroll
+  for (int j = 0; j < KP; ++j) {
+    const bool sw = better(v, id, vals[j], ids[j]);
+    const float tv = vals[j];
+    const int ti = ids[j];
+    vals[j] = sw ? v : tv;
+    ids[j] = sw ? id : ti;
+    v = sw ? tv : v;
+    id = sw ? ti : id;
+  }
+}
+
+template <int KP>
+__device__ __forceinline__ void list_clear(float (&vals)[KP], int (&ids)[KP]) {
+#pragma unroll
+  for (int j = 0; j < KP; ++j) {
+    vals[j] = -INFINITY;
+    ids[j] = INVALID_ID;
+  }
+}
+
+// Warp-wide extraction of the best `kout` entries of 32 sorted lists. Lane r < kout ends
+// holding the r-th best in (out_v, out_i).
+template <int KP>
+__device__ __forceinline__ void warp_extract(float (&vals)[KP], int (&ids)[KP], int kout,
+                                             float& out_v, int& out_i) {
+  const int lane = threadIdx.x & 31;
+  out_v = -INFINITY;
+  out_i = INVALID_ID;
+  for (int r = 0; r < kout; ++r) {
+    float bv = vals[0];
+    int bi = ids[0];
+#pragma unroll
+    for (int off = 16; off; off >>= 1) {
+      const float ov = __shfl_xor_sync(FULL_MASK, bv, off);
+      const int oi = __shfl_xor_sync(FULL_MASK, bi, off);
+      if (better(ov, oi, bv, bi)) {
+        bv = ov;
+        bi = oi;
+      }
+    }
+    const bool win = (ids[0] == bi) && (vals[0] == bv);
+#pragma unroll
+    for (int j = 0; j < KP - 1; ++j) {
+      vals[j] = win ? vals[j + 1] : vals[j];
+      ids[j] = win ? ids[j + 1] : ids[j];
+    }
+    if (win) {
+      vals[KP - 1] = -INFINITY;
+      ids[KP - 1] = INVALID_ID;
+    }
+    if (lane == r) {
+      out_v = bv;
+      out_i = bi;
+    }
+  }
+}
+
+__device__ __forceinline__ float warp_sum(float x) {
+#pragma unroll
+  for (int off = 16; off; off >>= 1) x += __shfl_xor_sync(FULL_MASK, x, off);
+  return x;
+}
+__device__ __forceinline__ float warp_max(float x) {
+#pragma unroll
+  for (int off = 16; off; off >>= 1) x = fmaxf(x, __shfl_xor_sync(FULL_MASK, x, off));
+  return x;
+}
+
+// Combine per-lane (max, sum of exp(x - max)) pairs into the warp's pair.
+__device__ __forceinline__ void warp_lse_combine(float& m, float& s) {
+  const float M = warp_max(m);
+  float t = (m == -INFINITY) ? 0.f : s * ex2((m - M) * LOG2E);
+  t = warp_sum(t);
+  m = M;
+  s = t;
+}
+
+__device__ __forceinline__ void set_status(int32_t* status, int code) {
+  if (status) atomicCAS(status, 0, code);
+}
+
+__device__ __forceinline__ float sigmoidf_(float x) { return 1.f / (1.f + expf(-x)); }
+
+// ---------------------------------------------------------------- sweep
+struct SweepSeg {
+  const void* logits;     // [rows, V]
+  int rows;               // rows in this segment
+  int kout;               // entries to output per row (K for proposal rows, 1 for verifier rows)
+  int32_t* out_ids;       // [rows, kout]
+  float* out_logprob;     // [rows, kout] or nullptr
+  float* out_lse;         // [rows]
+  float* part_val;        // [rows, nchunk, KP]
+  int32_t* part_id;       // [rows, nchunk, KP]
+  float* part_m;          // [rows, nchunk]
+  float* part_s;          // [rows, nchunk]
+  int32_t* counters;      // [rows]
+};
+
+struct SweepLaunch {
+  SweepSeg seg[2];
+  int nseg;
+  int V;
+  int nchunk;
+  int KP;
+  int dtype;              // brisk_dtype of the logits
+  int32_t* status;
+};
+
+int sweep_chunks(int rows_per_tensor, int V, int dtype, int num_sms);
+int kp_for(int K);
+cudaError_t launch_sweep(const SweepLaunch& a, cudaStream_t stream);
+
+// ---------------------------------------------------------------- dense products (SIMT, fp32 accumulate)
+// C[m, n] = sum_k A(m, k) B(n, k), A(m,k) = A[m*lda + k], B(n,k) = transB ? B[k*ldb + n] : B[n*ldb + k].
+cudaError_t gemm_simt(int M, int N, int K, const void* A, int a_dt, int lda, const void* B,
+                      int b_dt, int ldb, bool transB, float* C, int ldc, cudaStream_t stream);
+// dst[i*ldd + j] = (dst type) src[i*lds + j], i < rows, j < cols.
+cudaError_t copy2d(int rows, int cols, const void* src, int s_dt, int lds, void* dst, int d_dt,
+                   int ldd, cudaStream_t stream);
+
+// ---------------------------------------------------------------- corrector scan and verify
+struct ScanArgs {
+  int B, L, V, K, S, logits_dt;
+  int select_mode, verify_mode;
+  int do_select, do_verify;
+  // corrector inputs
+  const void* logits_q;
+  const int32_t* cand_ids;
+  const float* cand_logprob;
+  const int32_t* x0;
+  const float* u_sel;
+  const float* G;        // [B*L, 2S] hidden-state part of the GRU pre-activations (z | h)
+  const float* G0;       // [B, S]    hidden-state part of Init
+  const float* Tzh;      // [V, 2S]   token part of the GRU pre-activations (z | h)
+  const float* U;        // [V, S]    residual rows: d = <s, U[c]>
+  const float* T0;       // [V, S]    token part of Init
+  const float* posz;     // [L, S]
+  const float* posh;     // [L, S]
+  const float* Fz;       // [S, 5]
+  const float* Fh;       // [S, 5]
+  const float* wg;       // [S + 5]
+  float b_g, alpha;
+  // select outputs (or verify inputs when do_select == 0)
+  int32_t* sel_tokens;   // [B, L]
+  float* refined;        // [B, L, K]
+  // verify inputs / outputs
+  const void* logits_p;
+  const int32_t* argmax_p;  // [B, L]
+  const float* lse_p;       // [B, L]
+  const float* u_acc;
+  const float* u_res;
+  int32_t* accepted_len;
+  int32_t* out_tokens;
+  int32_t* correction;
+  int32_t* next_anchor;
+  int32_t* status;
+};
+
+size_t scan_smem_bytes(int L, int K, int S, int V);
+cudaError_t launch_scan(const ScanArgs& a, cudaStream_t stream);
+
+}  // namespace brisk

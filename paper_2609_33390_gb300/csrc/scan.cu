@@ -1,0 +1,492 @@
+// Corrector scan and verification, one CTA per sequence.
+//
+// Corrector (Sec. 3.3 Eqs. 4-5; App. C.2 Eq. 7; Algorithm 1(b) loop). The
+// minimal-GRU pre-activations are linear in the input blocks
+// [P_h m_i ; P_e E_in(x_{i-1}) ; pos_i ; P_phi phi_i], so each block's share is
+// read from a precomputed source:
+//   hidden share   G[b,i]          (one dense product over all b, i, before the scan)
+//   token share    Tzh[x_{i-1}]    (vocabulary table folded once per weight set)
+//   position share posz[i], posh[i]
+//   feature share  Fz phi_i, Fh phi_i   (S x 5 folded matrices)
+// and the residual d_{i,k} = <W_s s_i, W_c E_out(c)> = <s_i, U[c]> with
+// U = (E_out W_c^T) W_s. Init is u_0 = tanh(G0[b] + T0[x0]). What stays
+// sequential per position is O(S) element work, K+1 dot products of length S
+// and the K-way Select.
+//
+// Verification (Sec. 3.1; Sec. 3.3; App. B Eq. 8) runs in the same CTA after
+// the scan, or alone (brisk_verify_block), through the same device code.
+#include "brisk_internal.cuh"
+
+namespace brisk {
+
+namespace {
+
+constexpr int SCAN_THREADS = 128;
+constexpr int SCAN_WARPS = SCAN_THREADS / 32;
+constexpr int EPT_MAX = 8;      // state elements per thread: S <= 1024
+constexpr int KMAX = 32;
+
+struct Smem {
+  float* s;        // [S]     state
+  float* F;        // [10][S] Fz then Fh, feature-major
+  float* d;        // [2][KMAX] residual dots (double-buffered)
+  float* gpart;    // [2][SCAN_WARPS] gate partial sums
+  int* cid;        // [L][K]
+  float* clp;      // [L][K]
+  float* top;      // [L][3]  l_i(c_0), l_i(c_1), l_i(c_3)
+  float* lprev;    // [L][K]  l_i(c_{i-1,k}); row 0 holds l_0(x0) in slot 0
+  int* sel;        // [L]
+  int* rank;       // [L]
+  float* ref;      // [L][K]
+  float* bsum;     // [nblk]  residual block sums
+  float* misc;     // [16]
+  int* imisc;      // [16]
+};
+
+__host__ __device__ inline size_t align16(size_t x) { return (x + 15) & ~size_t(15); }
+
+constexpr int RES_BLOCK = 256;  // residual-sampling block: 32 lanes x 8 ids
+
+__host__ __device__ inline size_t smem_layout(int L, int K, int S, int V, char* base, Smem* sm) {
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    const size_t o = off;
+    off = align16(off + bytes);
+    return base ? base + o : nullptr;
+  };
+  const int nblk = (V + RES_BLOCK - 1) / RES_BLOCK;
+  char* p_s = take(sizeof(float) * S);
+  char* p_F = take(sizeof(float) * 10 * S);
+  char* p_d = take(sizeof(float) * 2 * KMAX);
+  char* p_g = take(sizeof(float) * 2 * SCAN_WARPS);
+  char* p_cid = take(sizeof(int) * L * K);
+  char* p_clp = take(sizeof(float) * L * K);
+  char* p_top = take(sizeof(float) * L * 3);
+  char* p_lprev = take(sizeof(float) * L * K);
+  char* p_sel = take(sizeof(int) * L);
+  char* p_rank = take(sizeof(int) * L);
+  char* p_ref = take(sizeof(float) * L * K);
+  char* p_bsum = take(sizeof(float) * nblk);
+  char* p_misc = take(sizeof(float) * 16);
+  char* p_imisc = take(sizeof(int) * 16);
+  if (sm) {
+    sm->s = (float*)p_s; sm->F = (float*)p_F; sm->d = (float*)p_d; sm->gpart = (float*)p_g;
+    sm->cid = (int*)p_cid; sm->clp = (float*)p_clp; sm->top = (float*)p_top;
+    sm->lprev = (float*)p_lprev; sm->sel = (int*)p_sel; sm->rank = (int*)p_rank;
+    sm->ref = (float*)p_ref; sm->bsum = (float*)p_bsum; sm->misc = (float*)p_misc;
+    sm->imisc = (int*)p_imisc;
+  }
+  return off;
+}
+
+__device__ __forceinline__ float load_logit(const void* base, int dt, size_t idx) {
+  if (dt == BRISK_DT_BF16) return __bfloat162float(reinterpret_cast<const __nv_bfloat16*>(base)[idx]);
+  return reinterpret_cast<const float*>(base)[idx];
+}
+
+// Select over the K refined scores of one position (identical in every thread).
+__device__ __forceinline__ int select_rank(const float* ref, int K, int mode, float u) {
+  if (mode == BRISK_SELECT_GREEDY) {
+    int best = 0;
+    float bv = ref[0];
+    for (int k = 1; k < K; ++k)
+      if (ref[k] > bv) { bv = ref[k]; best = k; }
+    return best;
+  }
+  float mx = ref[0];
+  for (int k = 1; k < K; ++k) mx = fmaxf(mx, ref[k]);
+  float tot = 0.f;
+  for (int k = 0; k < K; ++k) tot += expf(ref[k] - mx);
+  const float target = u * tot;
+  float cum = 0.f;
+  int last = 0;
+  for (int k = 0; k < K; ++k) {
+    const float w = expf(ref[k] - mx);
+    cum += w;
+    if (w > 0.f) last = k;
+    if (cum > target) return k;
+  }
+  return last;
+}
+
+// pi_i(rank r) of the proposal law induced by the Select rule.
+__device__ __forceinline__ float proposal_mass(const float* ref, int K, int mode, int r) {
+  if (mode == BRISK_SELECT_GREEDY) return 1.f;
+  float mx = ref[0];
+  for (int k = 1; k < K; ++k) mx = fmaxf(mx, ref[k]);
+  float tot = 0.f;
+  for (int k = 0; k < K; ++k) tot += expf(ref[k] - mx);
+  return expf(ref[r] - mx) / tot;
+}
+
+// Residual R(v) = max(0, p(v) - pi(v)) of the 8 ids [v0, v0+8) owned by this lane.
+// Lanes k < K hold candidate k: (cand_id, cand_mass).
+__device__ __forceinline__ void residual8(const void* rowp, int dt, int V, float lse, int v0,
+                                         int blk0, int cand_id, float cand_mass, int K,
+                                         float (&R)[8]) {
+  const int lane = threadIdx.x & 31;
+#pragma unroll
+  for (int e = 0; e < 8; ++e) {
+    const int v = v0 + e;
+    R[e] = (v < V) ? expf(load_logit(rowp, dt, (size_t)v) - lse) : 0.f;
+  }
+  const bool mine = lane < K && cand_id >= blk0 && cand_id < blk0 + RES_BLOCK;
+  unsigned mask = __ballot_sync(FULL_MASK, mine);
+  while (mask) {
+    const int k = __ffs(mask) - 1;
+    mask &= mask - 1;
+    const int cid = __shfl_sync(FULL_MASK, cand_id, k);
+    const float cm = __shfl_sync(FULL_MASK, cand_mass, k);
+    const int rel = cid - v0;
+#pragma unroll
+    for (int e = 0; e < 8; ++e)
+      if (rel == e) R[e] -= cm;
+  }
+#pragma unroll
+  for (int e = 0; e < 8; ++e) R[e] = fmaxf(R[e], 0.f);
+}
+
+// Draw from the normalised [p - pi]_+ of verifier row `rowp` with uniform u, walking ids in
+// ascending order; the verifier argmax when the residual mass is <= RESID_Z_FLOOR. CTA-wide.
+__device__ int residual_sample(const Smem& sm, const void* rowp, int dt, int V, float lse,
+                               const int* cid, const float* ref, int K, int select_mode,
+                               int sel_rank, float u, int argmax_p) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int nblk = (V + RES_BLOCK - 1) / RES_BLOCK;
+  // candidate k's proposal mass, held by lane k
+  int cand_id = -1;
+  float cand_mass = 0.f;
+  if (lane < K) {
+    cand_id = cid[lane];
+    if (select_mode == BRISK_SELECT_GREEDY) cand_mass = (lane == sel_rank) ? 1.f : 0.f;
+    else cand_mass = proposal_mass(ref, K, select_mode, lane);
+  }
+  // pass 1: block sums (blocks interleaved over warps)
+  for (int blk = warp; blk < nblk; blk += SCAN_WARPS) {
+    const int blk0 = blk * RES_BLOCK;
+    float R[8];
+    residual8(rowp, dt, V, lse, blk0 + lane * 8, blk0, cand_id, cand_mass, K, R);
+    float t = 0.f;
+#pragma unroll
+    for (int e = 0; e < 8; ++e) t += R[e];
+    t = warp_sum(t);
+    if (lane == 0) sm.bsum[blk] = t;
+  }
+  __syncthreads();
+  // warp 0: total mass and the block holding the target
+  if (warp == 0) {
+    const int per = (nblk + 31) / 32;
+    const int b0 = lane * per, b1 = min(nblk, b0 + per);
+    float mine = 0.f;
+    for (int b = b0; b < b1; ++b) mine += sm.bsum[b];
+    float incl = mine;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const float o = __shfl_up_sync(FULL_MASK, incl, off);
+      if (lane >= off) incl += o;
+    }
+    const float Z = __shfl_sync(FULL_MASK, incl, 31);
+    const float target = u * Z;
+    int found = -1;
+    float before = 0.f;
+    // first lane whose run holds the target, then the block inside the run
+    const unsigned hit = __ballot_sync(FULL_MASK, incl > target && b1 > b0);
+    if (hit) {
+      const int l = __ffs(hit) - 1;
+      if (lane == l) {
+        float acc = incl - mine;
+        for (int b = b0; b < b1; ++b) {
+          if (acc + sm.bsum[b] > target) { found = b; break; }
+          acc += sm.bsum[b];
+        }
+        if (found < 0) found = b1 - 1;
+        before = acc;
+        sm.imisc[0] = found;
+        sm.imisc[3] = 0;
+        sm.misc[0] = before;
+      }
+    } else if (lane == 0) {
+      // rounding put the target at or past the end: the last id with mass
+      int lastb = -1;
+      for (int b = nblk - 1; b >= 0; --b)
+        if (sm.bsum[b] > 0.f) { lastb = b; break; }
+      sm.imisc[0] = lastb;
+      sm.imisc[3] = 1;
+      sm.misc[0] = 0.f;
+    }
+    if (lane == 0) {
+      sm.misc[1] = Z;
+      sm.misc[2] = target;
+    }
+  }
+  __syncthreads();
+  const float Z = sm.misc[1];
+  if (!(Z > RESID_Z_FLOOR)) return argmax_p;
+  const int blk = sm.imisc[0];
+  if (blk < 0) return argmax_p;
+  // warp 0 walks the block: lane prefix sums, then the lane's 8 ids in order
+  if (warp == 0) {
+    const int blk0 = blk * RES_BLOCK;
+    float R[8];
+    residual8(rowp, dt, V, lse, blk0 + lane * 8, blk0, cand_id, cand_mass, K, R);
+    float mine = 0.f;
+#pragma unroll
+    for (int e = 0; e < 8; ++e) mine += R[e];
+    float incl = mine;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const float o = __shfl_up_sync(FULL_MASK, incl, off);
+      if (lane >= off) incl += o;
+    }
+    const float before = sm.misc[0];
+    const float target = sm.misc[2];
+    const bool past_end = sm.imisc[3] != 0;
+    const unsigned hit = past_end ? 0u : __ballot_sync(FULL_MASK, before + incl > target);
+    int pick = -1;
+    if (hit) {
+      const int l = __ffs(hit) - 1;
+      if (lane == l) {
+        float acc = before + incl - mine;
+        int lastpos = -1;
+        for (int e = 0; e < 8; ++e) {
+          if (R[e] > 0.f) lastpos = e;
+          acc += R[e];
+          if (acc > target) { pick = blk0 + lane * 8 + e; break; }
+        }
+        if (pick < 0) pick = blk0 + lane * 8 + (lastpos < 0 ? 0 : lastpos);
+      }
+      pick = __shfl_sync(FULL_MASK, pick, l);
+    } else {
+      // the last id of the block with positive residual
+      const unsigned pos = __ballot_sync(FULL_MASK, mine > 0.f);
+      if (pos) {
+        const int l = 31 - __clz(pos);
+        if (lane == l) {
+          int lastpos = 0;
+          for (int e = 0; e < 8; ++e)
+            if (R[e] > 0.f) lastpos = e;
+          pick = blk0 + lane * 8 + lastpos;
+        }
+        pick = __shfl_sync(FULL_MASK, pick, l);
+      } else {
+        pick = argmax_p;
+      }
+    }
+    if (lane == 0) sm.imisc[1] = pick;
+  }
+  __syncthreads();
+  return sm.imisc[1];
+}
+
+// Left-to-right verification of sm.sel against the verifier rows of sequence b.
+__device__ void verify_sequence(const ScanArgs& a, const Smem& sm, int b) {
+  const int tid = threadIdx.x;
+  const int L = a.L, K = a.K;
+  if (tid == 0) sm.imisc[2] = L;
+  __syncthreads();
+  for (int t = tid; t < L; t += SCAN_THREADS) {
+    const size_t bi = (size_t)b * L + t;
+    const int x = sm.sel[t];
+    bool ok;
+    if (a.verify_mode == BRISK_VERIFY_GREEDY) {
+      ok = (x == a.argmax_p[bi]);
+    } else {
+      const float lpx = load_logit(a.logits_p, a.logits_dt, bi * a.V + x);
+      const float px = expf(lpx - a.lse_p[bi]);
+      const float pim = proposal_mass(sm.ref + (size_t)t * K, K, a.select_mode, sm.rank[t]);
+      const float alpha = fminf(1.f, px / pim);
+      ok = a.u_acc[bi] < alpha;
+    }
+    if (!ok) atomicMin(&sm.imisc[2], t);
+  }
+  __syncthreads();
+  const int j = sm.imisc[2];
+  int corr = -1;
+  if (j < L) {
+    const size_t bj = (size_t)b * L + j;
+    if (a.verify_mode == BRISK_VERIFY_GREEDY) {
+      corr = a.argmax_p[bj];
+    } else {
+      const void* rowp = (a.logits_dt == BRISK_DT_BF16)
+                             ? (const void*)(reinterpret_cast<const __nv_bfloat16*>(a.logits_p) + bj * a.V)
+                             : (const void*)(reinterpret_cast<const float*>(a.logits_p) + bj * a.V);
+      corr = residual_sample(sm, rowp, a.logits_dt, a.V, a.lse_p[bj], sm.cid + (size_t)j * K,
+                             sm.ref + (size_t)j * K, K, a.select_mode, sm.rank[j], a.u_res[bj],
+                             a.argmax_p[bj]);
+    }
+  }
+  if (tid == 0) {
+    a.accepted_len[b] = j;
+    a.correction[b] = (j < L) ? corr : -1;
+    if (a.next_anchor) a.next_anchor[b] = (j < L) ? corr : sm.sel[L - 1];
+  }
+  for (int t = tid; t < L; t += SCAN_THREADS)
+    a.out_tokens[(size_t)b * L + t] = t < j ? sm.sel[t] : (t == j ? corr : -1);
+}
+
+__global__ void __launch_bounds__(SCAN_THREADS)
+scan_kernel(const __grid_constant__ ScanArgs a) {
+  extern __shared__ __align__(16) char smem_raw[];
+  Smem sm;
+  smem_layout(a.L, a.K, a.S, a.V, smem_raw, &sm);
+  const int b = blockIdx.x;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int L = a.L, K = a.K, S = a.S, V = a.V;
+  const size_t bL = (size_t)b * L;
+
+  // Ids are gathered with below, so out-of-range ones (a row with no finite logit leaves
+  // placeholder ids; caller-provided ids may be anything) are replaced by 0 and reported.
+  for (int e = tid; e < L * K; e += SCAN_THREADS) {
+    int c = a.cand_ids[bL * K + e];
+    if (c < 0 || c >= V) { set_status(a.status, BRISK_ERR_NUMERIC); c = 0; }
+    sm.cid[e] = c;
+  }
+  if (a.do_select) {
+    for (int e = tid; e < L * K; e += SCAN_THREADS) sm.clp[e] = a.cand_logprob[bL * K + e];
+  } else {
+    for (int e = tid; e < L * K; e += SCAN_THREADS) sm.ref[e] = a.refined[bL * K + e];
+    for (int e = tid; e < L; e += SCAN_THREADS) {
+      int x = a.sel_tokens[bL + e];
+      if (x < 0 || x >= V) { set_status(a.status, BRISK_ERR_INVALID_ARG); x = 0; }
+      sm.sel[e] = x;
+    }
+  }
+  __syncthreads();
+
+  if (a.do_select) {
+    int x0 = a.x0[b];
+    if (x0 < 0 || x0 >= V) {
+      if (tid == 0) set_status(a.status, BRISK_ERR_INVALID_ARG);
+      x0 = 0;
+    }
+    // features' logit gathers, all independent of the selections
+    for (int e = tid; e < L * 3; e += SCAN_THREADS) {
+      const int i = e / 3, w = e % 3;
+      const int c = sm.cid[i * K + (w == 0 ? 0 : (w == 1 ? 1 : 3))];
+      sm.top[e] = load_logit(a.logits_q, a.logits_dt, (bL + i) * V + c);
+    }
+    for (int e = tid; e < L * K; e += SCAN_THREADS) {
+      const int i = e / K, k = e % K;
+      float v = 0.f;
+      if (i == 0) { if (k == 0) v = load_logit(a.logits_q, a.logits_dt, bL * V + x0); }
+      else v = load_logit(a.logits_q, a.logits_dt, (bL + i) * V + sm.cid[(i - 1) * K + k]);
+      sm.lprev[e] = v;
+    }
+    for (int e = tid; e < 5 * S; e += SCAN_THREADS) {
+      const int j = e / 5, f = e % 5;
+      sm.F[f * S + j] = a.Fz[e];
+      sm.F[(5 + f) * S + j] = a.Fh[e];
+    }
+    float s[EPT_MAX], wg[EPT_MAX];
+#pragma unroll
+    for (int q = 0; q < EPT_MAX; ++q) {
+      const int j = tid + q * SCAN_THREADS;
+      s[q] = 0.f;
+      wg[q] = 0.f;
+      if (j < S) {
+        s[q] = tanhf(a.G0[(size_t)b * S + j] + a.T0[(size_t)x0 * S + j]);
+        wg[q] = a.wg[j];
+      }
+    }
+    float wgf[5];
+#pragma unroll
+    for (int f = 0; f < 5; ++f) wgf[f] = a.wg[S + f];
+    const float sig_alpha = sigmoidf_(a.alpha);
+    __syncthreads();
+
+    int prev = x0, prank = 0;
+    for (int i = 0; i < L; ++i) {
+      const int buf = i & 1;
+      const int* ci = sm.cid + i * K;
+      // confidence features of position i (App. C.2)
+      const float l0 = sm.top[i * 3 + 0];
+      float phi[5];
+      phi[0] = l0 - sm.top[i * 3 + 1];
+      phi[1] = l0 - sm.top[i * 3 + 2];
+      phi[2] = (prev == ci[0]) ? 1.f : 0.f;
+      phi[3] = (prev == ci[0] || prev == ci[1] || prev == ci[2] || prev == ci[3]) ? 1.f : 0.f;
+      phi[4] = l0 - sm.lprev[i * K + (i == 0 ? 0 : prank)];
+      // minimal-GRU step on this thread's state elements
+      const float* Gi = a.G + (bL + i) * 2 * S;
+      const float* Ti = a.Tzh + (size_t)prev * 2 * S;
+      float gacc = 0.f;
+#pragma unroll
+      for (int q = 0; q < EPT_MAX; ++q) {
+        const int j = tid + q * SCAN_THREADS;
+        if (j < S) {
+          float zp = Gi[j] + a.posz[(size_t)i * S + j] + Ti[j];
+          float hp = Gi[S + j] + a.posh[(size_t)i * S + j] + Ti[S + j];
+#pragma unroll
+          for (int f = 0; f < 5; ++f) {
+            zp = fmaf(sm.F[f * S + j], phi[f], zp);
+            hp = fmaf(sm.F[(5 + f) * S + j], phi[f], hp);
+          }
+          const float z = sigmoidf_(zp);
+          s[q] = (1.f - z) * s[q] + z * hp;
+          sm.s[j] = s[q];
+          gacc = fmaf(wg[q], s[q], gacc);
+        }
+      }
+      gacc = warp_sum(gacc);
+      if (lane == 0) sm.gpart[buf * SCAN_WARPS + warp] = gacc;
+      __syncthreads();
+      // residual dots d_k = <s, U[c_k]>, one warp per candidate
+      for (int k = warp; k < K; k += SCAN_WARPS) {
+        const float* Uc = a.U + (size_t)ci[k] * S;
+        float acc = 0.f;
+        for (int j = lane; j < S; j += 32) acc = fmaf(sm.s[j], Uc[j], acc);
+        acc = warp_sum(acc);
+        if (lane == 0) sm.d[buf * KMAX + k] = acc;
+      }
+      __syncthreads();
+      // gate, refined scores and Select (every thread, identical arithmetic)
+      float gate = a.b_g;
+      for (int w = 0; w < SCAN_WARPS; ++w) gate += sm.gpart[buf * SCAN_WARPS + w];
+#pragma unroll
+      for (int f = 0; f < 5; ++f) gate = fmaf(wgf[f], phi[f], gate);
+      const float gamma = sig_alpha * sigmoidf_(gate);
+      float ref[KMAX];
+      for (int k = 0; k < K; ++k) ref[k] = sm.clp[i * K + k] + gamma * sm.d[buf * KMAX + k];
+      const float u = (a.select_mode == BRISK_SELECT_SAMPLE) ? a.u_sel[bL + i] : 0.f;
+      const int pick = select_rank(ref, K, a.select_mode, u);
+      if (tid < K) {
+        sm.ref[i * K + tid] = ref[tid];
+        a.refined[(bL + i) * K + tid] = ref[tid];
+      }
+      prank = pick;
+      prev = ci[pick];
+      if (tid == 0) {
+        sm.sel[i] = prev;
+        sm.rank[i] = pick;
+        a.sel_tokens[bL + i] = prev;
+      }
+    }
+    __syncthreads();
+  } else {
+    // verify alone: recover each selection's rank in its candidate list
+    for (int i = tid; i < L; i += SCAN_THREADS) {
+      int r = 0;
+      for (int k = 0; k < K; ++k)
+        if (sm.cid[i * K + k] == sm.sel[i]) { r = k; break; }
+      sm.rank[i] = r;
+    }
+    __syncthreads();
+  }
+
+  if (a.do_verify) verify_sequence(a, sm, b);
+}
+
+}  // namespace
+
+size_t scan_smem_bytes(int L, int K, int S, int V) { return smem_layout(L, K, S, V, nullptr, nullptr); }
+
+cudaError_t launch_scan(const ScanArgs& a, cudaStream_t stream) {
+  const size_t smem = scan_smem_bytes(a.L, a.K, a.S, a.V);
+  cudaError_t e = cudaFuncSetAttribute(scan_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)smem);
+  if (e != cudaSuccess) return e;
+  scan_kernel<<<a.B, SCAN_THREADS, smem, stream>>>(a);
+  return cudaGetLastError();
+}
+
+}  // namespace brisk

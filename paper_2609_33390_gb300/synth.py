@@ -125,13 +125,15 @@ def philox_words(keys: Sequence[int], stream: int, start: int, count: int, devic
     return words[:, off:off + count]
 
 
-_CHUNK_WORDS = 1 << 22
+def _chunk_words(device) -> int:
+    """Philox words generated per slab: bounded host memory, fewer launches on a GPU."""
+    return (1 << 26) if torch.device(device).type == "cuda" else (1 << 22)
 
 
 def _draw(keys, stream, count, device, fn, out_dtype=torch.float64, words_per_item=1):
     """Apply ``fn`` to consecutive word groups in bounded chunks; returns [len(keys), count]."""
     out = torch.empty((len(keys), count), dtype=out_dtype, device=device)
-    per = max(1, _CHUNK_WORDS // max(1, len(keys)) // words_per_item)
+    per = max(1, _chunk_words(device) // max(1, len(keys)) // words_per_item)
     for s in range(0, count, per):
         n = min(per, count - s)
         w = philox_words(keys, stream, s * words_per_item, n * words_per_item, device)
@@ -255,9 +257,8 @@ def weight_shapes(wl: Workload) -> dict:
     }
 
 
-def make_weights(wl: Workload, device="cpu", seed: Optional[int] = None) -> dict:
-    """Corrector parameters N(0, weight_std), frozen embedding rows E_in, E_out N(0, emb_std),
-    gate bias b_g = 0 and gate scale alpha = 0. Tensors are in ``wl.hidden_dtype``."""
+def make_corrector_weights(wl: Workload, device="cpu", seed: Optional[int] = None) -> dict:
+    """The corrector parameters alone, N(0, weight_std), in ``wl.hidden_dtype``."""
     seed = wl.seed if seed is None else seed
     key = [splitmix64(seed ^ _WEIGHT_KEY_SALT)]
     out = {}
@@ -265,9 +266,18 @@ def make_weights(wl: Workload, device="cpu", seed: Optional[int] = None) -> dict
         n = math.prod(shape)
         w = normal(key, S_W + j, n, device).view(shape) * wl.weight_std
         out[name] = w.to(wl.hidden_dtype)
+    return out
+
+
+def make_weights(wl: Workload, device="cpu", seed: Optional[int] = None) -> dict:
+    """Corrector parameters N(0, weight_std), frozen embedding rows E_in, E_out N(0, emb_std),
+    gate bias b_g = 0 and gate scale alpha = 0. Tensors are in ``wl.hidden_dtype``."""
+    seed = wl.seed if seed is None else seed
+    key = [splitmix64(seed ^ _WEIGHT_KEY_SALT)]
+    out = make_corrector_weights(wl, device, seed)
     for name, stream in (("E_in", S_EIN), ("E_out", S_EOUT)):
         e = torch.empty((wl.V, wl.d), dtype=wl.hidden_dtype, device=device)
-        rows = max(1, (1 << 23) // wl.d)
+        rows = max(1, _chunk_words(device) // (2 * wl.d))
         for v0 in range(0, wl.V, rows):
             nv = min(rows, wl.V - v0)
             z = _normal_range(key, stream, v0 * wl.d, nv * wl.d, device)
@@ -276,6 +286,29 @@ def make_weights(wl: Workload, device="cpu", seed: Optional[int] = None) -> dict
     out["b_g"] = 0.0
     out["alpha"] = 0.0
     return out
+
+
+class EmbeddingRows:
+    """Rows of E_in / E_out generated on demand, identical to ``make_weights``'s tensors
+    (for consumers that need a few rows of a large vocabulary table)."""
+
+    def __init__(self, wl: Workload, which: str, seed: Optional[int] = None):
+        seed = wl.seed if seed is None else seed
+        self.key = [splitmix64(seed ^ _WEIGHT_KEY_SALT)]
+        self.stream = S_EIN if which == "E_in" else S_EOUT
+        self.wl = wl
+        self.cache = {}
+
+    def row(self, v: int) -> torch.Tensor:
+        v = int(v)
+        if v not in self.cache:
+            d = self.wl.d
+            z = _normal_range(self.key, self.stream, v * d, d, "cpu") * self.wl.emb_std
+            self.cache[v] = z.to(self.wl.hidden_dtype)
+        return self.cache[v]
+
+    def __getitem__(self, v):
+        return self.row(v)
 
 
 def _normal_range(keys, stream, start, count, device):
@@ -353,7 +386,7 @@ def make_block(wl: Workload, device="cpu", seqs: Optional[Iterable[int]] = None,
     keys = [sequence_key(seed, s, block) for s in seqs]
     agree = agreement(wl_s, seqs, device)
     if chunk <= 0:
-        chunk = max(1, (1 << 24) // max(1, wl.L * wl.V))
+        chunk = max(1, (_chunk_words(device) // 4) // max(1, wl.L * wl.V))
     lq = torch.empty((n, wl.L, wl.V), dtype=wl.logits_dtype, device=device)
     lp = torch.empty_like(lq)
     for c in range(0, n, chunk):
