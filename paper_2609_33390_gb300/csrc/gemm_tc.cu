@@ -1,0 +1,325 @@
+// Tensor-core product C[m, n] = sum_k A[m, k] B[n, k] for bf16 A, B (both K-contiguous)
+// with fp32 accumulation, on the 5th-generation tensor cores of sm_103a.
+//
+// One CTA computes one 128 x BN tile. A TMA producer thread streams 64-wide K
+// slices of A and B into a 4-stage ring of 128-byte-swizzled shared-memory
+// buffers; one thread issues tcgen05.mma (M = 128, N = BN, K = 16) into a TMEM
+// accumulator and releases each stage with tcgen05.commit; then all four warps
+// read their 32 TMEM lanes back with tcgen05.ld and write the tile. Every
+// wait on an mbarrier is bounded: on expiry the CTA records BRISK_ERR_TIMEOUT,
+// drains what it started and frees its TMEM.
+//
+// Used for the corrector's one dense contraction (the MASK hidden states times
+// the hidden projection, App. C.2 "64-dimensional projection of the MASK
+// hidden state") and for the products that follow it, where an fp32 operand
+// enters as the sum of two bf16 parts (hi + lo) so that bf16 tensor cores keep
+// fp32-level accuracy.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include "brisk_internal.cuh"
+
+namespace brisk {
+
+namespace {
+
+constexpr int TC_BM = 128;
+constexpr int TC_BK = 64;               // one 128-byte swizzle row of bf16
+constexpr int TC_STAGES = 4;
+constexpr int TC_THREADS = 128;
+constexpr uint64_t WAIT_LIMIT_NS = 2000000000ull;   // 2 s per wait
+
+__device__ __forceinline__ uint32_t su32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ uint64_t gtimer() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(su32(bar)), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(su32(bar)), "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(su32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+// Bounded wait for the phase with the given parity; false on expiry or abort.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag) {
+  const uint64_t t0 = gtimer();
+  while (!mbar_try_wait(bar, parity)) {
+    if (*abort_flag) return false;
+    if (gtimer() - t0 > WAIT_LIMIT_NS) return false;
+  }
+  return true;
+}
+__device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, uint64_t* bar, int x,
+                                            int y) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%3, %4}], [%2];" ::"r"(su32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(su32(bar)), "r"(x), "r"(y)
+      : "memory");
+}
+__device__ __forceinline__ void tmem_alloc(uint32_t* slot, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(su32(slot)),
+               "r"(ncols)
+               : "memory");
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
+               : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+// D(tmem) (+)= A(smem desc) * B(smem desc)^T, kind::f16 (bf16 inputs), fp32 accumulator.
+__device__ __forceinline__ void umma(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                     uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(tmem_d),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+__device__ __forceinline__ void umma_commit(uint64_t* bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(su32(bar))
+      : "memory");
+}
+// 32 lanes x 8 consecutive fp32 columns of TMEM, waited for before returning.
+__device__ __forceinline__ void tmem_ld8(uint32_t taddr, float (&v)[8]) {
+  uint32_t r0, r1, r2, r3, r4, r5, r6, r7;
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];\n\t"
+      "tcgen05.wait::ld.sync.aligned;"
+      : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3), "=r"(r4), "=r"(r5), "=r"(r6), "=r"(r7)
+      : "r"(taddr)
+      : "memory");
+  v[0] = __uint_as_float(r0); v[1] = __uint_as_float(r1); v[2] = __uint_as_float(r2);
+  v[3] = __uint_as_float(r3); v[4] = __uint_as_float(r4); v[5] = __uint_as_float(r5);
+  v[6] = __uint_as_float(r6); v[7] = __uint_as_float(r7);
+}
+
+// Shared-memory matrix descriptor of a K-major tile stored as 8-row x 128-byte
+// swizzle atoms (the layout TMA writes with 128-byte swizzling): start address,
+// leading offset 16 B (unused by this layout), 1024 B between 8-row groups,
+// descriptor version 1, swizzle mode 128 B.
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
+  uint64_t d = 0;
+  d |= static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4);
+  d |= static_cast<uint64_t>(16 >> 4) << 16;
+  d |= static_cast<uint64_t>(1024 >> 4) << 32;
+  d |= static_cast<uint64_t>(1) << 46;
+  d |= static_cast<uint64_t>(2) << 61;
+  return d;
+}
+
+// Instruction descriptor of kind::f16: fp32 accumulator, bf16 A and B, both K-major, M x N.
+__host__ __device__ constexpr uint32_t idesc_bf16(int M, int N) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | (static_cast<uint32_t>(N >> 3) << 17) |
+         (static_cast<uint32_t>(M >> 4) << 24);
+}
+
+struct TcArgs {
+  int M, N, K;
+  int BN;           // tile columns (multiple of 16, <= 256)
+  int tmem_cols;    // power of two >= max(32, BN)
+  int mode;         // 0: fp32 C[m*ldc + n]; 1: bf16 hi at [m*ldc + n], lo at [m*ldc + N + n]
+  int ldc;
+  void* C;
+  int32_t* status;
+};
+
+__global__ void __launch_bounds__(TC_THREADS, 1)
+gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+               const TcArgs a) {
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  // 1024-byte alignment of every stage buffer (required by the 128-byte swizzle atoms)
+  uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  const int a_bytes = TC_BM * TC_BK * 2;
+  const int b_bytes = a.BN * TC_BK * 2;
+  uint8_t* sA = base;
+  uint8_t* sB = base + TC_STAGES * a_bytes;
+  uint64_t* full = reinterpret_cast<uint64_t*>(sB + TC_STAGES * b_bytes);
+  uint64_t* empty = full + TC_STAGES;
+  uint64_t* accum = empty + TC_STAGES;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(accum + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int m0 = blockIdx.x * TC_BM, n0 = blockIdx.y * a.BN;
+  const int nk = (a.K + TC_BK - 1) / TC_BK;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < TC_STAGES; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    mbar_init(accum, 1);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 0) tmem_alloc(tmem_slot, a.tmem_cols);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  int issued = 0;    // stages the producer started (for draining on abort)
+  if (warp == 0 && lane == 0) {
+    // TMA producer
+    for (int kb = 0; kb < nk; ++kb) {
+      const int s = kb % TC_STAGES;
+      if (kb >= TC_STAGES && !mbar_wait(&empty[s], ((kb / TC_STAGES) & 1) ^ 1, abort_flag)) {
+        *abort_flag = 1;
+        break;
+      }
+      mbar_expect_tx(&full[s], a_bytes + b_bytes);
+      tma_load_2d(sA + s * a_bytes, &tmA, &full[s], kb * TC_BK, m0);
+      tma_load_2d(sB + s * b_bytes, &tmB, &full[s], kb * TC_BK, n0);
+      issued = kb + 1;
+    }
+  } else if (warp == 1 && lane == 0) {
+    // MMA issuer
+    const uint32_t idesc = idesc_bf16(TC_BM, a.BN);
+    for (int kb = 0; kb < nk; ++kb) {
+      const int s = kb % TC_STAGES;
+      if (!mbar_wait(&full[s], (kb / TC_STAGES) & 1, abort_flag)) {
+        *abort_flag = 1;
+        break;
+      }
+      tc_fence_after();
+      const uint64_t ad = sw128_desc(su32(sA + s * a_bytes));
+      const uint64_t bd = sw128_desc(su32(sB + s * b_bytes));
+#pragma unroll
+      for (int kk = 0; kk < TC_BK / 16; ++kk)   // 16 bf16 = 32 bytes per step: +2 in 16-byte units
+        umma(tmem, ad + 2 * kk, bd + 2 * kk, idesc, (kb > 0 || kk > 0) ? 1u : 0u);
+      umma_commit(&empty[s]);
+    }
+    umma_commit(accum);
+  }
+  __syncwarp();
+
+  // epilogue: every warp owns TMEM lanes [32*warp, 32*warp + 32) = tile rows
+  const bool ok = mbar_wait(accum, 0, abort_flag);
+  tc_fence_after();
+  if (ok && !*abort_flag) {
+    const int row = m0 + warp * 32 + lane;
+    const uint32_t trow = tmem + (static_cast<uint32_t>(warp * 32) << 16);
+    for (int c = 0; c < a.BN; c += 8) {
+      float v[8];
+      tmem_ld8(trow + c, v);
+      if (row < a.M) {
+        if (a.mode == 0) {
+          float* C = static_cast<float*>(a.C) + (size_t)row * a.ldc;
+#pragma unroll
+          for (int j = 0; j < 8; ++j)
+            if (n0 + c + j < a.N) C[n0 + c + j] = v[j];
+        } else {
+          __nv_bfloat16* C = static_cast<__nv_bfloat16*>(a.C) + (size_t)row * a.ldc;
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            const int n = n0 + c + j;
+            if (n < a.N) {
+              const __nv_bfloat16 hi = __float2bfloat16_rn(v[j]);
+              C[n] = hi;
+              C[a.N + n] = __float2bfloat16_rn(v[j] - __bfloat162float(hi));
+            }
+          }
+        }
+      }
+    }
+  } else if (threadIdx.x == 0) {
+    set_status(a.status, BRISK_ERR_TIMEOUT);
+    *abort_flag = 1;
+  }
+  // drain: the producer's loads complete on their own; wait (bounded) for the ones issued
+  if (warp == 0 && lane == 0 && *abort_flag) {
+    for (int kb = (issued > TC_STAGES ? issued - TC_STAGES : 0); kb < issued; ++kb) {
+      const uint64_t t0 = gtimer();
+      while (!mbar_try_wait(&full[kb % TC_STAGES], (kb / TC_STAGES) & 1) &&
+             gtimer() - t0 < WAIT_LIMIT_NS) {
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) tmem_dealloc(tmem, a.tmem_cols);
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  }
+  return fn;
+}
+
+// 2-D bf16 tensor [rows, cols] with row stride ld (elements), boxes of 64 x box_rows, 128-byte swizzle.
+bool make_map(CUtensorMap* map, const void* ptr, int rows, int cols, int ld, int box_rows) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows)};
+  cuuint64_t strides[1] = {static_cast<cuuint64_t>(ld) * 2};
+  cuuint32_t box[2] = {static_cast<cuuint32_t>(TC_BK), static_cast<cuuint32_t>(box_rows)};
+  cuuint32_t estr[2] = {1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+}  // namespace
+
+size_t gemm_tc_smem(int BN) {
+  return 1024 + TC_STAGES * (TC_BM * TC_BK * 2 + BN * TC_BK * 2) + (2 * TC_STAGES + 1) * 8 + 16;
+}
+
+bool gemm_tc_supported(const void* A, int lda, const void* B, int ldb, int K) {
+  return encode_fn() != nullptr && (reinterpret_cast<uintptr_t>(A) % 16 == 0) &&
+         (reinterpret_cast<uintptr_t>(B) % 16 == 0) && (lda % 8 == 0) && (ldb % 8 == 0) && K >= 1;
+}
+
+// C = A B^T with A [M, K] (row stride lda) and B [N, K] (row stride ldb), bf16, fp32 accumulate.
+cudaError_t gemm_tc(int M, int N, int K, const void* A, int lda, const void* B, int ldb, int mode,
+                    void* C, int ldc, int32_t* status, cudaStream_t stream) {
+  if (M <= 0 || N <= 0) return cudaSuccess;
+  int BN = ((N + 15) / 16) * 16;
+  if (BN > 256) BN = 256;
+  int cols = 32;
+  while (cols < BN) cols *= 2;
+  CUtensorMap ta, tb;
+  if (!make_map(&ta, A, M, K, lda, TC_BM) || !make_map(&tb, B, N, K, ldb, BN))
+    return cudaErrorInvalidValue;
+  TcArgs a{M, N, K, BN, cols, mode, ldc, C, status};
+  const size_t smem = gemm_tc_smem(BN);
+  cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       static_cast<int>(smem));
+  if (e != cudaSuccess) return e;
+  const dim3 grid((M + TC_BM - 1) / TC_BM, (N + BN - 1) / BN);
+  gemm_tc_kernel<<<grid, TC_THREADS, smem, stream>>>(ta, tb, a);
+  return cudaGetLastError();
+}
+
+}  // namespace brisk
