@@ -443,6 +443,30 @@ def run_e2e(args, tail, pool, wl, sm, vm, dev):
             "steps": n, "ms_per_step": 1000.0 * secs / n, "_tokens": acc, "_seconds": secs}
 
 
+def run_profile(args):
+    """A short run for profilers: `--steps` fused decode-tail calls on one block of the named
+    workload (no timing output). Used to capture single kernels under ncu."""
+    import torch
+    from paper_2609_33390_gb300 import build, brisk, synth
+    build.build()
+    dev = torch.device("cuda")
+    wl = synth.WORKLOADS[args.profile]
+    weights = synth.make_weights(wl, dev)
+    tail = brisk.DecodeTail.for_workload(wl, weights, dev)
+    tail.prepare()
+    blk = synth.make_block(wl, dev)
+    sm, vm = brisk.mode_ids(wl.select_mode, wl.verify_mode)
+    out = tail.alloc_outputs(full=False)
+    for _ in range(args.warmup + args.steps):
+        tail.tail(blk, sm, vm, out=out)
+    torch.cuda.synchronize()
+    st = tail.device_status()
+    print(json.dumps({"profile": args.profile, "calls": args.warmup + args.steps,
+                      "status": brisk.status_string(st),
+                      "accepted": int(out["accepted_len"].sum())}))
+    return 0 if st == brisk.OK else 1
+
+
 def main(argv=None):
     ap = argparse.ArgumentParser(description=__doc__.splitlines()[0])
     ap.add_argument("--gpus", type=int, default=1)
@@ -452,8 +476,11 @@ def main(argv=None):
     ap.add_argument("--pool", type=int, default=16, help="distinct pre-generated blocks cycled")
     ap.add_argument("--e2e-steps", type=int, default=20)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--profile", default=None, help="workload name: short untimed run for ncu")
     args = ap.parse_args(argv)
     args.warmup = max(3, args.warmup)   # at least 3 untimed warm-up steps
+    if args.profile:
+        return run_profile(args)
     if args.impl == "reference":
         return run_reference(args)
     return run_ours(args)

@@ -113,7 +113,7 @@ typedef struct brisk_tail_io {
   int32_t *sel_tokens;      /* optional [B, L]    selected tokens x_i                     */
   float *refined;           /* optional [B, L, K] refined scores                          */
   int32_t *accepted_len;    /* [B]    accepted prefix length a, 0..L                      */
-  int32_t *out_tokens;      /* [B, L] x_0..x_{a-1}, then the correction at a (if a < L), then -1 */
+  int32_t *out_tokens;      /* [B, L] sel_tokens[0..a-1], the correction at a (if a < L), then -1 */
   int32_t *correction;      /* [B]    correction token, -1 when a == L                    */
   int32_t *next_anchor;     /* optional [B] last committed token (anchor of the next block) */
 } brisk_tail_io;
