@@ -147,6 +147,25 @@ brisk_status brisk_topk_candidates(const brisk_dims *dims, const void *logits_q,
                                    int32_t *cand_ids, float *cand_logprob, float *lse_q,
                                    void *workspace, void *stream);
 
+/* Step 1 for callers that cannot allocate device memory. The paper has no counterpart; this
+ * is a deployment variant of brisk_topk_candidates with the same inputs, outputs and results
+ * but no workspace argument. Some callers cannot hand the library a workspace: a plug-in that
+ * runs inside another runtime and only receives its input and output buffers, an engine whose
+ * memory manager owns all of HBM and forbids ad-hoc cudaMalloc, a decode loop that must not
+ * allocate. This entry point keeps its scratch in a fixed 4 MiB array inside the library,
+ * present on every GPU that loads the library until the process exits, and allocates nothing.
+ *  - Returns BRISK_ERR_UNSUPPORTED when the problem needs more than that array holds (its
+ *    per-row arrival counters and per-chunk partial results grow with B*L and K).
+ *  - The first call on a device looks up the array's device address (cudaGetSymbolAddress);
+ *    make that first call before any stream capture.
+ *  - Every call on a device shares the one array; calls that can overlap on the GPU (other
+ *    streams, other host threads) race and must be serialised by the caller.
+ *  - Device-side problems are not reported through a status word: a row without a finite
+ *    logit shows as a non-finite lse_q. */
+brisk_status brisk_topk_candidates_noalloc(const brisk_dims *dims, const void *logits_q,
+                                           int32_t *cand_ids, float *cand_logprob, float *lse_q,
+                                           void *stream);
+
 /* Step 2 (Sec. 3.3 Eqs. 4-5; App. C.2 Eq. 7; Algorithm 1(b) loop): per sequence, sequentially
  * over positions, the minimal-GRU corrector state, the gated low-rank residual on the K
  * candidates and Select. Reads the step-1 outputs (cand_ids, cand_logprob) and logits_q

@@ -70,6 +70,8 @@ _SIGS = [
     ("brisk_decode_tail", ctypes.c_int,
      [ctypes.POINTER(Dims), ctypes.POINTER(Params), _vp, ctypes.POINTER(TailIO), ctypes.c_int32,
       ctypes.c_int32, _vp, ctypes.POINTER(Events), _vp]),
+    ("brisk_topk_candidates_noalloc", ctypes.c_int,
+     [ctypes.POINTER(Dims), _vp, _vp, _vp, _vp, _vp]),
     ("brisk_kernels_per_tail", ctypes.c_int32, [ctypes.POINTER(Dims)]),
     ("brisk_last_device_status", ctypes.c_int, [_vp, ctypes.c_int32, _vp]),
     ("brisk_status_string", ctypes.c_char_p, [ctypes.c_int]),
@@ -136,6 +138,13 @@ def tables_bytes(dims: Dims) -> int:
 
 def kernels_per_tail(dims: Dims) -> int:
     return int(lib().brisk_kernels_per_tail(ctypes.byref(dims)))
+
+
+def topk_candidates_noalloc(dims: Dims, logits_q, cand_ids, cand_logprob, lse_q, stream=None) -> int:
+    """Step 1 without a workspace, for callers that cannot allocate device memory; the
+    library's own fixed scratch array is used instead. Returns the status code."""
+    return int(lib().brisk_topk_candidates_noalloc(ctypes.byref(dims), _p(logits_q), _p(cand_ids),
+                                                   _p(cand_logprob), _p(lse_q), _stream(stream)))
 
 
 def make_params(w: Dict[str, object]) -> Params:
