@@ -54,7 +54,7 @@ WsLayout ws_layout(const brisk_dims* d) {
   w.lse_q = take(sizeof(float) * BL);
   w.sel = take(sizeof(int32_t) * BL);
   w.refined = take(sizeof(float) * BL * d->K);
-  w.Hm = take(sizeof(float) * (BL + d->B) * d->r);
+  w.Hm = take(6 * (BL + d->B) * d->r);   // fp32 [BL+B, r] or bf16 [BL+B, 3r]
   w.G = take(sizeof(float) * BL * 2 * S);
   w.G0 = take(sizeof(float) * d->B * S);
   w.total = o;
@@ -67,11 +67,13 @@ WsLayout ws_layout(const brisk_dims* d) {
 // U   [V, S] : residual rows, U(v) = W_s^T W_c E_out(v)
 // T0  [V, S] : token share of Init, W0[:, r:2r] P_e E_in(v)
 // Tin, Tout [V, r]: P_e E_in(v), W_c E_out(v) (intermediates of the folds)
-// posz, posh [L, S]: position shares W_z[:, 2r:2r+16] pos_i, W_h[:, 2r:2r+16] pos_i
+// posG [L, 2S]: position shares W_z[:, 2r:2r+16] pos_i | W_h[:, 2r:2r+16] pos_i (added to G)
 // Fz, Fh [S, 5]: feature shares W_z[:, 2r+16:] P_phi, W_h[:, 2r+16:] P_phi
 // wg [S+5] fp32 copy of w_g; W2 [2S, r] = [W_z[:, :r] ; W_h[:, :r]] and W0h [S, r] = W0[:, :r] (fp32)
+// W2s [2S, 3r], W0s [S, 3r] (bf16): the same blocks written three times along k, so that
+// [hi | mid | lo] W^T = (hi + mid + lo) W^T on bf16 tensor cores.
 struct TbLayout {
-  size_t Tzh, U, T0, Tin, Tout, posz, posh, Fz, Fh, wg, W2, W0h, total;
+  size_t Tzh, U, T0, Tin, Tout, posG, Fz, Fh, wg, W2, W0h, W2s, W0s, total;
 };
 
 TbLayout tb_layout(const brisk_dims* d) {
@@ -84,13 +86,14 @@ TbLayout tb_layout(const brisk_dims* d) {
   t.T0 = take(sizeof(float) * V * S);
   t.Tin = take(sizeof(float) * V * r);
   t.Tout = take(sizeof(float) * V * r);
-  t.posz = take(sizeof(float) * L * S);
-  t.posh = take(sizeof(float) * L * S);
+  t.posG = take(sizeof(float) * L * 2 * S);
   t.Fz = take(sizeof(float) * S * 5);
   t.Fh = take(sizeof(float) * S * 5);
   t.wg = take(sizeof(float) * (S + 5));
   t.W2 = take(sizeof(float) * 2 * S * r);
   t.W0h = take(sizeof(float) * S * r);
+  t.W2s = take(2 * 2 * S * 3 * r);
+  t.W0s = take(2 * S * 3 * r);
   t.total = o;
   return t;
 }
@@ -140,18 +143,37 @@ SweepSeg make_seg(const WsLayout& w, void* ws, int seg, const void* logits, int 
 }
 
 // The hidden-state shares of the corrector: Hm = [hidden ; h_ctx] P_h^T, then
-// G = Hm[:BL] [W_z[:, :r] ; W_h[:, :r]]^T and G0 = Hm[BL:] W0[:, :r]^T.
+// G = Hm[:BL] [W_z[:, :r] ; W_h[:, :r]]^T and G0 = Hm[BL:] W0[:, :r]^T. With bf16 weights the
+// products run on the tensor cores: the first one writes Hm as three bf16 parts, which the
+// second one multiplies by the weight blocks written three times along k (fp32-level accuracy).
 brisk_status hidden_products(const brisk_dims* d, const brisk_params* p, const void* tables,
                              const void* hidden, const void* h_ctx, const WsLayout& w, void* ws,
                              cudaStream_t st) {
   const TbLayout t = tb_layout(d);
   const int BL = d->B * d->L, r = d->r, S = 2 * d->r, hd = d->hidden_dtype;
+  int32_t* status = at<int32_t>(ws, w.status);
+  if (hd == BRISK_DT_BF16 && gemm_tc_supported(hidden, d->d, p->P_h, d->d, d->d) &&
+      aligned(h_ctx, 16)) {
+    __nv_bfloat16* Hs = at<__nv_bfloat16>(ws, w.Hm);   // [BL + B, 3r]: hi | mid | lo
+    const int r3 = 3 * r;
+    const TcSpec first[2] = {
+        {BL, r, d->d, hidden, d->d, p->P_h, d->d, 1, Hs, r3, nullptr, 0},
+        {d->B, r, d->d, h_ctx, d->d, p->P_h, d->d, 1, Hs + (size_t)BL * r3, r3, nullptr, 0}};
+    BRISK_CUDA(gemm_tc_grouped(first, 2, status, st));
+    const TcSpec second[2] = {
+        {BL, 2 * S, r3, Hs, r3, at<__nv_bfloat16>(tables, t.W2s), r3, 0, at<float>(ws, w.G), 2 * S,
+         at<float>(tables, t.posG), d->L},
+        {d->B, S, r3, Hs + (size_t)BL * r3, r3, at<__nv_bfloat16>(tables, t.W0s), r3, 0,
+         at<float>(ws, w.G0), S, nullptr, 0}};
+    BRISK_CUDA(gemm_tc_grouped(second, 2, status, st));
+    return BRISK_OK;
+  }
   float* Hm = at<float>(ws, w.Hm);
   BRISK_CUDA(gemm_simt(BL, r, d->d, hidden, hd, d->d, p->P_h, hd, d->d, false, Hm, r, st));
   BRISK_CUDA(gemm_simt(d->B, r, d->d, h_ctx, hd, d->d, p->P_h, hd, d->d, false,
                        Hm + (size_t)BL * r, r, st));
   BRISK_CUDA(gemm_simt(BL, 2 * S, r, Hm, BRISK_DT_F32, r, at<float>(tables, t.W2), BRISK_DT_F32, r,
-                       false, at<float>(ws, w.G), 2 * S, st));
+                       false, at<float>(ws, w.G), 2 * S, st, at<float>(tables, t.posG), d->L));
   BRISK_CUDA(gemm_simt(d->B, S, r, Hm + (size_t)BL * r, BRISK_DT_F32, r, at<float>(tables, t.W0h),
                        BRISK_DT_F32, r, false, at<float>(ws, w.G0), S, st));
   return BRISK_OK;
@@ -167,8 +189,6 @@ ScanArgs scan_args(const brisk_dims* d, const brisk_params* p, const void* table
     a.Tzh = at<float>(tables, t.Tzh);
     a.U = at<float>(tables, t.U);
     a.T0 = at<float>(tables, t.T0);
-    a.posz = at<float>(tables, t.posz);
-    a.posh = at<float>(tables, t.posh);
     a.Fz = at<float>(tables, t.Fz);
     a.Fh = at<float>(tables, t.Fh);
     a.wg = at<float>(tables, t.wg);
@@ -236,9 +256,9 @@ brisk_status brisk_corrector_prepare(const brisk_dims* d, const brisk_params* p,
   BRISK_CUDA(gemm_simt(V, S, r, Tout, F32, r, p->W_s, hd, S, true, at<float>(tables, t.U), S, st));
   // position shares
   BRISK_CUDA(gemm_simt(L, S, 16, p->pos, hd, 16, wp(p->Wz, 2 * r), hd, ldw, false,
-                       at<float>(tables, t.posz), S, st));
+                       at<float>(tables, t.posG), 2 * S, st));
   BRISK_CUDA(gemm_simt(L, S, 16, p->pos, hd, 16, wp(p->Wh, 2 * r), hd, ldw, false,
-                       at<float>(tables, t.posh), S, st));
+                       at<float>(tables, t.posG) + S, 2 * S, st));
   // feature shares: F(j, f) = sum_t W[j, 2r+16+t] P_phi[t, f]
   BRISK_CUDA(gemm_simt(S, 5, 16, wp(p->Wz, 2 * r + 16), hd, ldw, p->P_phi, hd, 5, true,
                        at<float>(tables, t.Fz), 5, st));
@@ -249,6 +269,16 @@ brisk_status brisk_corrector_prepare(const brisk_dims* d, const brisk_params* p,
   BRISK_CUDA(copy2d(S, r, p->Wz, hd, ldw, at<float>(tables, t.W2), F32, r, st));
   BRISK_CUDA(copy2d(S, r, p->Wh, hd, ldw, at<float>(tables, t.W2) + (size_t)S * r, F32, r, st));
   BRISK_CUDA(copy2d(S, r, p->W0, hd, 2 * r, at<float>(tables, t.W0h), F32, r, st));
+  if (hd == BRISK_DT_BF16) {
+    const int BF = BRISK_DT_BF16;
+    __nv_bfloat16* W2s = at<__nv_bfloat16>(tables, t.W2s);
+    __nv_bfloat16* W0s = at<__nv_bfloat16>(tables, t.W0s);
+    for (int part = 0; part < 3; ++part) {
+      BRISK_CUDA(copy2d(S, r, p->Wz, hd, ldw, W2s + part * r, BF, 3 * r, st));
+      BRISK_CUDA(copy2d(S, r, p->Wh, hd, ldw, W2s + (size_t)S * 3 * r + part * r, BF, 3 * r, st));
+      BRISK_CUDA(copy2d(S, r, p->W0, hd, 2 * r, W0s + part * r, BF, 3 * r, st));
+    }
+  }
   return BRISK_OK;
 }
 
@@ -421,7 +451,8 @@ brisk_status brisk_decode_tail(const brisk_dims* d, const brisk_params* p, const
 
 int32_t brisk_kernels_per_tail(const brisk_dims* dims) {
   if (!dims_ok(dims)) return 0;
-  return 1 /* sweep */ + 4 /* hidden-state products */ + 1 /* scan + verify */;
+  const bool tc = dims->hidden_dtype == BRISK_DT_BF16;
+  return 1 /* sweep */ + (tc ? 2 : 4) /* hidden-state products */ + 1 /* scan + verify */;
 }
 
 brisk_status brisk_last_device_status(void* ws, int32_t clear, void* stream) {

@@ -179,7 +179,28 @@ cudaError_t launch_sweep(const SweepLaunch& a, cudaStream_t stream);
 // ---------------------------------------------------------------- dense products (SIMT, fp32 accumulate)
 // C[m, n] = sum_k A(m, k) B(n, k), A(m,k) = A[m*lda + k], B(n,k) = transB ? B[k*ldb + n] : B[n*ldb + k].
 cudaError_t gemm_simt(int M, int N, int K, const void* A, int a_dt, int lda, const void* B,
-                      int b_dt, int ldb, bool transB, float* C, int ldc, cudaStream_t stream);
+                      int b_dt, int ldb, bool transB, float* C, int ldc, cudaStream_t stream,
+                      const float* bias = nullptr, int bias_period = 1);
+// Tensor-core product on sm_103a: C = A B^T with A [M, K] and B [N, K] bf16 (row strides lda, ldb),
+// fp32 accumulation; mode 0 stores fp32 C[m*ldc + n], mode 1 stores three bf16 parts whose sum
+// is c to about 2^-24 relative (hi at [m*ldc + n], mid at [m*ldc + N + n], lo at [m*ldc + 2N + n]).
+cudaError_t gemm_tc(int M, int N, int K, const void* A, int lda, const void* B, int ldb, int mode,
+                    void* C, int ldc, int32_t* status, cudaStream_t stream);
+// Up to two independent products of the same kind in one launch.
+struct TcSpec {
+  int M, N, K;
+  const void* A;
+  int lda;
+  const void* B;
+  int ldb;
+  int mode;
+  void* C;
+  int ldc;
+  const float* bias;   // optional fp32 [bias_period, N] added to row m as bias[m % bias_period] (mode 0)
+  int bias_period;
+};
+cudaError_t gemm_tc_grouped(const TcSpec* spec, int nprob, int32_t* status, cudaStream_t stream);
+bool gemm_tc_supported(const void* A, int lda, const void* B, int ldb, int K);
 // dst[i*ldd + j] = (dst type) src[i*lds + j], i < rows, j < cols.
 cudaError_t copy2d(int rows, int cols, const void* src, int s_dt, int lds, void* dst, int d_dt,
                    int ldd, cudaStream_t stream);
@@ -189,19 +210,20 @@ struct ScanArgs {
   int B, L, V, K, S, logits_dt;
   int select_mode, verify_mode;
   int do_select, do_verify;
+  int ubuf;              // residual-row buffers in shared memory (set by launch_scan)
+  int tcand;             // token-share rows of the candidates staged in shared memory (set by launch_scan)
   // corrector inputs
   const void* logits_q;
   const int32_t* cand_ids;
   const float* cand_logprob;
   const int32_t* x0;
   const float* u_sel;
-  const float* G;        // [B*L, 2S] hidden-state part of the GRU pre-activations (z | h)
+  const float* G;        // [B*L, 2S] hidden and position shares of the GRU pre-activations (z | h)
   const float* G0;       // [B, S]    hidden-state part of Init
   const float* Tzh;      // [V, 2S]   token part of the GRU pre-activations (z | h)
   const float* U;        // [V, S]    residual rows: d = <s, U[c]>
   const float* T0;       // [V, S]    token part of Init
-  const float* posz;     // [L, S]
-  const float* posh;     // [L, S]
+
   const float* Fz;       // [S, 5]
   const float* Fh;       // [S, 5]
   const float* wg;       // [S + 5]

@@ -13,7 +13,8 @@ constexpr int TM = 64, TN = 64, TK = 16;
 template <typename TA, typename TB>
 __global__ void __launch_bounds__(256)
 gemm_simt_kernel(int M, int N, int K, const TA* __restrict__ A, int lda,
-                 const TB* __restrict__ B, int ldb, int transB, float* __restrict__ C, int ldc) {
+                 const TB* __restrict__ B, int ldb, int transB, float* __restrict__ C, int ldc,
+                 const float* __restrict__ bias, int bias_period) {
   __shared__ float As[TK][TM + 4];
   __shared__ float Bs[TK][TN + 4];
   const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
@@ -61,7 +62,7 @@ gemm_simt_kernel(int M, int N, int K, const TA* __restrict__ A, int lda,
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
       const long long gn = n0 + tx * 4 + j;
-      if (gn < N) C[gm * ldc + gn] = acc[i][j];
+      if (gn < N) C[gm * ldc + gn] = acc[i][j] + (bias ? bias[(gm % bias_period) * N + gn] : 0.f);
     }
   }
 }
@@ -81,10 +82,12 @@ __global__ void copy2d_kernel(int rows, int cols, const TS* __restrict__ src, in
 
 template <typename TA, typename TB>
 cudaError_t gemm_t(int M, int N, int K, const void* A, int lda, const void* B, int ldb,
-                   bool transB, float* C, int ldc, cudaStream_t stream) {
+                   bool transB, float* C, int ldc, cudaStream_t stream, const float* bias,
+                   int bias_period) {
   const dim3 grid((N + TN - 1) / TN, (M + TM - 1) / TM);
   gemm_simt_kernel<TA, TB><<<grid, 256, 0, stream>>>(
-      M, N, K, static_cast<const TA*>(A), lda, static_cast<const TB*>(B), ldb, transB ? 1 : 0, C, ldc);
+      M, N, K, static_cast<const TA*>(A), lda, static_cast<const TB*>(B), ldb, transB ? 1 : 0, C, ldc,
+      bias, bias_period > 0 ? bias_period : 1);
   return cudaGetLastError();
 }
 
@@ -105,15 +108,19 @@ cudaError_t copy_t(int rows, int cols, const void* src, int lds, void* dst, int 
 }  // namespace
 
 cudaError_t gemm_simt(int M, int N, int K, const void* A, int a_dt, int lda, const void* B,
-                      int b_dt, int ldb, bool transB, float* C, int ldc, cudaStream_t stream) {
+                      int b_dt, int ldb, bool transB, float* C, int ldc, cudaStream_t stream,
+                      const float* bias, int bias_period) {
   if (M <= 0 || N <= 0) return cudaSuccess;
   if (a_dt == BRISK_DT_BF16 && b_dt == BRISK_DT_BF16)
-    return gemm_t<__nv_bfloat16, __nv_bfloat16>(M, N, K, A, lda, B, ldb, transB, C, ldc, stream);
+    return gemm_t<__nv_bfloat16, __nv_bfloat16>(M, N, K, A, lda, B, ldb, transB, C, ldc, stream,
+                                                 bias, bias_period);
   if (a_dt == BRISK_DT_F32 && b_dt == BRISK_DT_BF16)
-    return gemm_t<float, __nv_bfloat16>(M, N, K, A, lda, B, ldb, transB, C, ldc, stream);
+    return gemm_t<float, __nv_bfloat16>(M, N, K, A, lda, B, ldb, transB, C, ldc, stream, bias,
+                                        bias_period);
   if (a_dt == BRISK_DT_BF16 && b_dt == BRISK_DT_F32)
-    return gemm_t<__nv_bfloat16, float>(M, N, K, A, lda, B, ldb, transB, C, ldc, stream);
-  return gemm_t<float, float>(M, N, K, A, lda, B, ldb, transB, C, ldc, stream);
+    return gemm_t<__nv_bfloat16, float>(M, N, K, A, lda, B, ldb, transB, C, ldc, stream, bias,
+                                        bias_period);
+  return gemm_t<float, float>(M, N, K, A, lda, B, ldb, transB, C, ldc, stream, bias, bias_period);
 }
 
 cudaError_t copy2d(int rows, int cols, const void* src, int s_dt, int lds, void* dst, int d_dt,

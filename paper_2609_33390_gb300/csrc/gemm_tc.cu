@@ -6,14 +6,14 @@
 // buffers; one thread issues tcgen05.mma (M = 128, N = BN, K = 16) into a TMEM
 // accumulator and releases each stage with tcgen05.commit; then all four warps
 // read their 32 TMEM lanes back with tcgen05.ld and write the tile. Every
-// wait on an mbarrier is bounded: on expiry the CTA records BRISK_ERR_TIMEOUT,
+// wait on an mbarrier is bounded (about 2 s of SM clock): on expiry the CTA records BRISK_ERR_TIMEOUT,
 // drains what it started and frees its TMEM.
 //
 // Used for the corrector's one dense contraction (the MASK hidden states times
 // the hidden projection, App. C.2 "64-dimensional projection of the MASK
 // hidden state") and for the products that follow it, where an fp32 operand
-// enters as the sum of two bf16 parts (hi + lo) so that bf16 tensor cores keep
-// fp32-level accuracy.
+// enters as the sum of three bf16 parts (hi + mid + lo) so that bf16 tensor
+// cores keep fp32-level accuracy.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -27,16 +27,12 @@ constexpr int TC_BM = 128;
 constexpr int TC_BK = 64;               // one 128-byte swizzle row of bf16
 constexpr int TC_STAGES = 4;
 constexpr int TC_THREADS = 128;
-constexpr uint64_t WAIT_LIMIT_NS = 2000000000ull;   // 2 s per wait
+constexpr long long WAIT_LIMIT_CYCLES = 4000000000ll;   // about 2 s of SM clock per wait
 
 __device__ __forceinline__ uint32_t su32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }
-__device__ __forceinline__ uint64_t gtimer() {
-  uint64_t t;
-  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-  return t;
-}
+
 __device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
   asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(su32(bar)), "r"(count) : "memory");
 }
@@ -55,14 +51,15 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
       : "memory");
   return ok != 0;
 }
-// Bounded wait for the phase with the given parity; false on expiry or abort.
+// Bounded wait for the phase with the given parity; false on expiry or abort. The SM cycle
+// counter and the abort flag are only read every 64 polls.
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag) {
-  const uint64_t t0 = gtimer();
-  while (!mbar_try_wait(bar, parity)) {
-    if (*abort_flag) return false;
-    if (gtimer() - t0 > WAIT_LIMIT_NS) return false;
+  if (mbar_try_wait(bar, parity)) return true;
+  const long long t0 = clock64();
+  for (unsigned n = 1;; ++n) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if ((n & 63) == 0 && (*abort_flag || clock64() - t0 > WAIT_LIMIT_CYCLES)) return false;
   }
-  return true;
 }
 __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, uint64_t* bar, int x,
                                             int y) {
@@ -103,18 +100,22 @@ __device__ __forceinline__ void umma_commit(uint64_t* bar) {
       "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(su32(bar))
       : "memory");
 }
-// 32 lanes x 8 consecutive fp32 columns of TMEM, waited for before returning.
-__device__ __forceinline__ void tmem_ld8(uint32_t taddr, float (&v)[8]) {
-  uint32_t r0, r1, r2, r3, r4, r5, r6, r7;
+// 32 lanes x 32 consecutive fp32 columns of TMEM, waited for before returning.
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
+  uint32_t r[32];
   asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];\n\t"
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,"
+      "%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];\n\t"
       "tcgen05.wait::ld.sync.aligned;"
-      : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3), "=r"(r4), "=r"(r5), "=r"(r6), "=r"(r7)
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]),
+        "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]),
+        "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
       : "r"(taddr)
       : "memory");
-  v[0] = __uint_as_float(r0); v[1] = __uint_as_float(r1); v[2] = __uint_as_float(r2);
-  v[3] = __uint_as_float(r3); v[4] = __uint_as_float(r4); v[5] = __uint_as_float(r5);
-  v[6] = __uint_as_float(r6); v[7] = __uint_as_float(r7);
+#pragma unroll
+  for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
 }
 
 // Shared-memory matrix descriptor of a K-major tile stored as 8-row x 128-byte
@@ -137,19 +138,29 @@ __host__ __device__ constexpr uint32_t idesc_bf16(int M, int N) {
          (static_cast<uint32_t>(M >> 4) << 24);
 }
 
-struct TcArgs {
+struct TcProblem {
   int M, N, K;
-  int BN;           // tile columns (multiple of 16, <= 256)
-  int tmem_cols;    // power of two >= max(32, BN)
-  int mode;         // 0: fp32 C[m*ldc + n]; 1: bf16 hi at [m*ldc + n], lo at [m*ldc + N + n]
+  int mode;         // 0: fp32 C[m*ldc + n]; 1: bf16 parts hi, mid, lo at [m*ldc + {0, N, 2N} + n]
   int ldc;
+  int mtiles, ntiles;
   void* C;
+  const float* bias;   // optional fp32 [bias_period, N], added to row m as bias[m % bias_period]
+  int bias_period;
+};
+
+struct TcArgs {
+  TcProblem p[2];   // one launch serves up to two independent products (grouped)
+  int nprob;
+  int tiles0;       // CTAs of problem 0
+  int BN;           // tile columns (multiple of 16, <= 256), shared by both problems
+  int tmem_cols;    // power of two >= max(32, BN)
   int32_t* status;
 };
 
 __global__ void __launch_bounds__(TC_THREADS, 1)
-gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-               const TcArgs a) {
+gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__ CUtensorMap tmB0,
+               const __grid_constant__ CUtensorMap tmA1, const __grid_constant__ CUtensorMap tmB1,
+               const __grid_constant__ TcArgs a) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   // 1024-byte alignment of every stage buffer (required by the 128-byte swizzle atoms)
   uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -164,8 +175,13 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int m0 = blockIdx.x * TC_BM, n0 = blockIdx.y * a.BN;
-  const int nk = (a.K + TC_BK - 1) / TC_BK;
+  const int pi = (a.nprob > 1 && (int)blockIdx.x >= a.tiles0) ? 1 : 0;
+  const TcProblem& P = a.p[pi];
+  const CUtensorMap* tmA = pi ? &tmA1 : &tmA0;
+  const CUtensorMap* tmB = pi ? &tmB1 : &tmB0;
+  const int tile = (int)blockIdx.x - (pi ? a.tiles0 : 0);
+  const int m0 = (tile % P.mtiles) * TC_BM, n0 = (tile / P.mtiles) * a.BN;
+  const int nk = (P.K + TC_BK - 1) / TC_BK;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < TC_STAGES; ++s) {
@@ -175,6 +191,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     mbar_init(accum, 1);
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
   }
   if (warp == 0) tmem_alloc(tmem_slot, a.tmem_cols);
   tc_fence_before();
@@ -192,8 +209,8 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         break;
       }
       mbar_expect_tx(&full[s], a_bytes + b_bytes);
-      tma_load_2d(sA + s * a_bytes, &tmA, &full[s], kb * TC_BK, m0);
-      tma_load_2d(sB + s * b_bytes, &tmB, &full[s], kb * TC_BK, n0);
+      tma_load_2d(sA + s * a_bytes, tmA, &full[s], kb * TC_BK, m0);
+      tma_load_2d(sB + s * b_bytes, tmB, &full[s], kb * TC_BK, n0);
       issued = kb + 1;
     }
   } else if (warp == 1 && lane == 0) {
@@ -215,47 +232,73 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     }
     umma_commit(accum);
   }
-  __syncwarp();
-
-  // epilogue: every warp owns TMEM lanes [32*warp, 32*warp + 32) = tile rows
-  const bool ok = mbar_wait(accum, 0, abort_flag);
+  // epilogue: one thread waits for the accumulator (with back-off, so that polling does not
+  // compete with TMA and the MMAs for the shared-memory pipe); the others wait at the barrier
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    const long long t0 = clock64();
+    bool done = false;
+    while (!(done = mbar_try_wait(accum, 0))) {
+      if (*abort_flag || clock64() - t0 > WAIT_LIMIT_CYCLES) break;
+      __nanosleep(128);
+    }
+    if (!done) *abort_flag = 1;
+  }
+  __syncthreads();
   tc_fence_after();
-  if (ok && !*abort_flag) {
-    const int row = m0 + warp * 32 + lane;
+  // Every warp owns TMEM lanes [32*warp, 32*warp + 32) = tile rows. Each 32 x 32 block goes
+  // through a padded shared-memory tile (the stage buffers are idle now) so that the global
+  // stores run along rows: one coalesced row segment per store instruction.
+  if (!*abort_flag) {
+    float* stage = reinterpret_cast<float*>(base) + warp * (32 * 33);
     const uint32_t trow = tmem + (static_cast<uint32_t>(warp * 32) << 16);
-    for (int c = 0; c < a.BN; c += 8) {
-      float v[8];
-      tmem_ld8(trow + c, v);
-      if (row < a.M) {
-        if (a.mode == 0) {
-          float* C = static_cast<float*>(a.C) + (size_t)row * a.ldc;
+    const int row0 = m0 + warp * 32;
+    for (int c0 = 0; c0 < a.BN; c0 += 32) {
+      float v[32];
+      tmem_ld32(trow + c0, v);
 #pragma unroll
-          for (int j = 0; j < 8; ++j)
-            if (n0 + c + j < a.N) C[n0 + c + j] = v[j];
+      for (int j = 0; j < 32; ++j) stage[lane * 33 + j] = v[j];
+      __syncwarp();
+      const int n = n0 + c0 + lane;
+      if (n < P.N) {
+        if (P.mode == 0) {
+          float* C = static_cast<float*>(P.C);
+          float bias[32];
+#pragma unroll
+          for (int rr = 0; rr < 32; ++rr)   // independent loads, all in flight before the stores
+            bias[rr] = (P.bias && row0 + rr < P.M)
+                           ? __ldg(P.bias + (size_t)((row0 + rr) % P.bias_period) * P.N + n)
+                           : 0.f;
+#pragma unroll
+          for (int rr = 0; rr < 32; ++rr)
+            if (row0 + rr < P.M) C[(size_t)(row0 + rr) * P.ldc + n] = stage[rr * 33 + lane] + bias[rr];
         } else {
-          __nv_bfloat16* C = static_cast<__nv_bfloat16*>(a.C) + (size_t)row * a.ldc;
-#pragma unroll
-          for (int j = 0; j < 8; ++j) {
-            const int n = n0 + c + j;
-            if (n < a.N) {
-              const __nv_bfloat16 hi = __float2bfloat16_rn(v[j]);
-              C[n] = hi;
-              C[a.N + n] = __float2bfloat16_rn(v[j] - __bfloat162float(hi));
-            }
+          __nv_bfloat16* C = static_cast<__nv_bfloat16*>(P.C);
+          for (int rr = 0; rr < 32 && row0 + rr < P.M; ++rr) {
+            // three bf16 parts, hi + mid + lo = x to about 2^-24 relative
+            const float x = stage[rr * 33 + lane];
+            const __nv_bfloat16 hi = __float2bfloat16_rn(x);
+            const float r1 = x - __bfloat162float(hi);
+            const __nv_bfloat16 mid = __float2bfloat16_rn(r1);
+            __nv_bfloat16* Cr = C + (size_t)(row0 + rr) * P.ldc;
+            Cr[n] = hi;
+            Cr[P.N + n] = mid;
+            Cr[2 * P.N + n] = __float2bfloat16_rn(r1 - __bfloat162float(mid));
           }
         }
       }
+      __syncwarp();
     }
-  } else if (threadIdx.x == 0) {
+  } else if (lane == 0) {
     set_status(a.status, BRISK_ERR_TIMEOUT);
     *abort_flag = 1;
   }
   // drain: the producer's loads complete on their own; wait (bounded) for the ones issued
   if (warp == 0 && lane == 0 && *abort_flag) {
     for (int kb = (issued > TC_STAGES ? issued - TC_STAGES : 0); kb < issued; ++kb) {
-      const uint64_t t0 = gtimer();
+      const long long t0 = clock64();
       while (!mbar_try_wait(&full[kb % TC_STAGES], (kb / TC_STAGES) & 1) &&
-             gtimer() - t0 < WAIT_LIMIT_NS) {
+             clock64() - t0 < WAIT_LIMIT_CYCLES) {
       }
     }
   }
@@ -301,25 +344,52 @@ bool gemm_tc_supported(const void* A, int lda, const void* B, int ldb, int K) {
          (reinterpret_cast<uintptr_t>(B) % 16 == 0) && (lda % 8 == 0) && (ldb % 8 == 0) && K >= 1;
 }
 
-// C = A B^T with A [M, K] (row stride lda) and B [N, K] (row stride ldb), bf16, fp32 accumulate.
-cudaError_t gemm_tc(int M, int N, int K, const void* A, int lda, const void* B, int ldb, int mode,
-                    void* C, int ldc, int32_t* status, cudaStream_t stream) {
-  if (M <= 0 || N <= 0) return cudaSuccess;
-  int BN = ((N + 15) / 16) * 16;
+// One or two products C = A B^T, A [M, K] (row stride lda) and B [N, K] (row stride ldb) bf16,
+// fp32 accumulation, in one launch.
+cudaError_t gemm_tc_grouped(const TcSpec* spec, int nprob, int32_t* status, cudaStream_t stream) {
+  if (nprob < 1 || nprob > 2) return cudaErrorInvalidValue;
+  int nmax = 0;
+  for (int i = 0; i < nprob; ++i) nmax = spec[i].N > nmax ? spec[i].N : nmax;
+  int BN = ((nmax + 15) / 16) * 16;
   if (BN > 256) BN = 256;
   int cols = 32;
   while (cols < BN) cols *= 2;
-  CUtensorMap ta, tb;
-  if (!make_map(&ta, A, M, K, lda, TC_BM) || !make_map(&tb, B, N, K, ldb, BN))
-    return cudaErrorInvalidValue;
-  TcArgs a{M, N, K, BN, cols, mode, ldc, C, status};
+  CUtensorMap maps[4];
+  TcArgs a{};
+  a.nprob = nprob;
+  a.BN = BN;
+  a.tmem_cols = cols;
+  a.status = status;
+  int total = 0;
+  for (int i = 0; i < 2; ++i) {
+    const TcSpec& q = spec[i < nprob ? i : 0];
+    if (!make_map(&maps[2 * i], q.A, q.M, q.K, q.lda, TC_BM) ||
+        !make_map(&maps[2 * i + 1], q.B, q.N, q.K, q.ldb, BN))
+      return cudaErrorInvalidValue;
+    if (i >= nprob) continue;
+    TcProblem& P = a.p[i];
+    P.M = q.M; P.N = q.N; P.K = q.K; P.mode = q.mode; P.ldc = q.ldc; P.C = q.C;
+    P.bias = q.bias;
+    P.bias_period = q.bias_period > 0 ? q.bias_period : 1;
+    P.mtiles = (q.M + TC_BM - 1) / TC_BM;
+    P.ntiles = (q.N + BN - 1) / BN;
+    if (i == 0) a.tiles0 = P.mtiles * P.ntiles;
+    total += P.mtiles * P.ntiles;
+  }
+  if (total == 0) return cudaSuccess;
   const size_t smem = gemm_tc_smem(BN);
   cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(smem));
   if (e != cudaSuccess) return e;
-  const dim3 grid((M + TC_BM - 1) / TC_BM, (N + BN - 1) / BN);
-  gemm_tc_kernel<<<grid, TC_THREADS, smem, stream>>>(ta, tb, a);
+  gemm_tc_kernel<<<total, TC_THREADS, smem, stream>>>(maps[0], maps[1], maps[2], maps[3], a);
   return cudaGetLastError();
+}
+
+cudaError_t gemm_tc(int M, int N, int K, const void* A, int lda, const void* B, int ldb, int mode,
+                    void* C, int ldc, int32_t* status, cudaStream_t stream) {
+  if (M <= 0 || N <= 0) return cudaSuccess;
+  const TcSpec s{M, N, K, A, lda, B, ldb, mode, C, ldc, nullptr, 0};
+  return gemm_tc_grouped(&s, 1, status, stream);
 }
 
 }  // namespace brisk

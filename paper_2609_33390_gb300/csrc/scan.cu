@@ -23,7 +23,7 @@ namespace {
 
 constexpr int SCAN_THREADS = 128;
 constexpr int SCAN_WARPS = SCAN_THREADS / 32;
-constexpr int EPT_MAX = 8;      // state elements per thread: S <= 1024
+constexpr int MCH = 2;          // 4-element state chunks per thread: S <= 4 * 128 * MCH = 1024
 constexpr int KMAX = 32;
 
 struct Smem {
@@ -41,13 +41,16 @@ struct Smem {
   float* bsum;     // [nblk]  residual block sums
   float* misc;     // [16]
   int* imisc;      // [16]
+  float* U;        // [ubuf][K][S] residual rows of the candidates (one or two positions)
+  float* Tc;       // [2][K][2S] token-share rows of a position's candidates (when they fit)
 };
 
 __host__ __device__ inline size_t align16(size_t x) { return (x + 15) & ~size_t(15); }
 
 constexpr int RES_BLOCK = 256;  // residual-sampling block: 32 lanes x 8 ids
 
-__host__ __device__ inline size_t smem_layout(int L, int K, int S, int V, char* base, Smem* sm) {
+__host__ __device__ inline size_t smem_layout(int L, int K, int S, int V, int ubuf, int tcand,
+                                              char* base, Smem* sm) {
   size_t off = 0;
   auto take = [&](size_t bytes) {
     const size_t o = off;
@@ -69,7 +72,11 @@ __host__ __device__ inline size_t smem_layout(int L, int K, int S, int V, char* 
   char* p_bsum = take(sizeof(float) * nblk);
   char* p_misc = take(sizeof(float) * 16);
   char* p_imisc = take(sizeof(int) * 16);
+  char* p_U = take(sizeof(float) * ubuf * K * S);
+  char* p_Tc = take(tcand ? sizeof(float) * 2 * K * 2 * S : 0);
   if (sm) {
+    sm->U = (float*)p_U;
+    sm->Tc = (float*)p_Tc;
     sm->s = (float*)p_s; sm->F = (float*)p_F; sm->d = (float*)p_d; sm->gpart = (float*)p_g;
     sm->cid = (int*)p_cid; sm->clp = (float*)p_clp; sm->top = (float*)p_top;
     sm->lprev = (float*)p_lprev; sm->sel = (int*)p_sel; sm->rank = (int*)p_rank;
@@ -79,29 +86,71 @@ __host__ __device__ inline size_t smem_layout(int L, int K, int S, int V, char* 
   return off;
 }
 
+__device__ __forceinline__ void cp_async16(void* smem, const void* gmem) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(
+                   static_cast<uint32_t>(__cvta_generic_to_shared(smem))),
+               "l"(gmem)
+               : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
+// Wait until at most n of this thread's most recent cp.async groups are still pending.
+__device__ __forceinline__ void cp_async_wait_pending(int n) {
+  if (n <= 0) asm volatile("cp.async.wait_group 0;" ::: "memory");
+  else if (n == 1) asm volatile("cp.async.wait_group 1;" ::: "memory");
+  else if (n == 2) asm volatile("cp.async.wait_group 2;" ::: "memory");
+  else asm volatile("cp.async.wait_group 3;" ::: "memory");
+}
+__device__ __forceinline__ float4 ld4(const float* p) { return *reinterpret_cast<const float4*>(p); }
+__device__ __forceinline__ void prefetch_l2(const void* p) {
+  asm volatile("prefetch.global.L2 [%0];" ::"l"(p));
+}
+
+// Residual rows U[c_k] of the K candidates into shared memory. Warp w owns candidates
+// k = w, w + 4, ...; lane l owns the 16-byte chunks l, l + 32, ... of each of its rows, and is
+// the only thread that later reads them, so its own cp.async wait suffices.
+__device__ __forceinline__ void fetch_U(float* Ush, const float* U, const int* ci, int K, int S) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  for (int k = warp; k < K; k += 4) {
+    const float* src = U + (size_t)ci[k] * S;
+    float* dst = Ush + (size_t)k * S;
+    for (int q = lane; q < S / 4; q += 32) cp_async16(dst + 4 * q, src + 4 * q);
+  }
+}
+// L2 prefetch of K vocabulary-table rows of `row_floats` floats.
+__device__ __forceinline__ void prefetch_rows(const float* table, const int* ci, int K, int row_floats) {
+  const int lines = (row_floats * 4 + 127) / 128;
+  for (int e = threadIdx.x; e < K * lines; e += SCAN_THREADS)
+    prefetch_l2(table + (size_t)ci[e / lines] * row_floats + (e % lines) * 32);
+}
+
 __device__ __forceinline__ float load_logit(const void* base, int dt, size_t idx) {
   if (dt == BRISK_DT_BF16) return __bfloat162float(reinterpret_cast<const __nv_bfloat16*>(base)[idx]);
   return reinterpret_cast<const float*>(base)[idx];
 }
 
-// Select over the K refined scores of one position (identical in every thread).
-__device__ __forceinline__ int select_rank(const float* ref, int K, int mode, float u) {
+// Select over the K refined scores of one position, refined_k = clp[k] + gamma * d[k] read from
+// shared memory (identical arithmetic in every thread).
+__device__ __forceinline__ int select_rank(const float* clp, const float* d, float gamma, int K,
+                                           int mode, float u) {
   if (mode == BRISK_SELECT_GREEDY) {
     int best = 0;
-    float bv = ref[0];
-    for (int k = 1; k < K; ++k)
-      if (ref[k] > bv) { bv = ref[k]; best = k; }
+    float bv = clp[0] + gamma * d[0];
+    for (int k = 1; k < K; ++k) {
+      const float v = clp[k] + gamma * d[k];
+      if (v > bv) { bv = v; best = k; }
+    }
     return best;
   }
-  float mx = ref[0];
-  for (int k = 1; k < K; ++k) mx = fmaxf(mx, ref[k]);
+  float mx = clp[0] + gamma * d[0];
+  for (int k = 1; k < K; ++k) mx = fmaxf(mx, clp[k] + gamma * d[k]);
   float tot = 0.f;
-  for (int k = 0; k < K; ++k) tot += expf(ref[k] - mx);
+  for (int k = 0; k < K; ++k) tot += expf(clp[k] + gamma * d[k] - mx);
   const float target = u * tot;
   float cum = 0.f;
   int last = 0;
   for (int k = 0; k < K; ++k) {
-    const float w = expf(ref[k] - mx);
+    const float w = expf(clp[k] + gamma * d[k] - mx);
     cum += w;
     if (w > 0.f) last = k;
     if (cum > target) return k;
@@ -328,7 +377,7 @@ __global__ void __launch_bounds__(SCAN_THREADS)
 scan_kernel(const __grid_constant__ ScanArgs a) {
   extern __shared__ __align__(16) char smem_raw[];
   Smem sm;
-  smem_layout(a.L, a.K, a.S, a.V, smem_raw, &sm);
+  smem_layout(a.L, a.K, a.S, a.V, a.ubuf, a.tcand, smem_raw, &sm);
   const int b = blockIdx.x;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int L = a.L, K = a.K, S = a.S, V = a.V;
@@ -377,27 +426,67 @@ scan_kernel(const __grid_constant__ ScanArgs a) {
       sm.F[f * S + j] = a.Fz[e];
       sm.F[(5 + f) * S + j] = a.Fh[e];
     }
-    float s[EPT_MAX], wg[EPT_MAX];
+    // this thread owns the 4-element state chunks c = tid + 128 m
+    const int nch = S / 4;
+    float4 s4[MCH], wg4[MCH], gz4[MCH], gh4[MCH], tz4[MCH], th4[MCH];
 #pragma unroll
-    for (int q = 0; q < EPT_MAX; ++q) {
-      const int j = tid + q * SCAN_THREADS;
-      s[q] = 0.f;
-      wg[q] = 0.f;
-      if (j < S) {
-        s[q] = tanhf(a.G0[(size_t)b * S + j] + a.T0[(size_t)x0 * S + j]);
-        wg[q] = a.wg[j];
+    for (int m = 0; m < MCH; ++m) {
+      const int c = tid + m * SCAN_THREADS;
+      s4[m] = wg4[m] = gz4[m] = gh4[m] = tz4[m] = th4[m] = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (c < nch) {
+        const float4 g0 = ld4(a.G0 + (size_t)b * S + 4 * c), t0 = ld4(a.T0 + (size_t)x0 * S + 4 * c);
+        s4[m] = make_float4(tanhf(g0.x + t0.x), tanhf(g0.y + t0.y), tanhf(g0.z + t0.z),
+                            tanhf(g0.w + t0.w));
+        wg4[m] = ld4(a.wg + 4 * c);
+        gz4[m] = ld4(a.G + bL * 2 * S + 4 * c);
+        gh4[m] = ld4(a.G + bL * 2 * S + S + 4 * c);
+        tz4[m] = ld4(a.Tzh + (size_t)x0 * 2 * S + 4 * c);        // token share of x_{-1} = x0
+        th4[m] = ld4(a.Tzh + (size_t)x0 * 2 * S + S + 4 * c);
       }
     }
     float wgf[5];
 #pragma unroll
     for (int f = 0; f < 5; ++f) wgf[f] = a.wg[S + f];
     const float sig_alpha = sigmoidf_(a.alpha);
+    // residual rows of positions 0 (and 1) into shared memory; one cp.async group per batch,
+    // committed even when empty, so that the group counts below are the same at every step
+    const int ubuf = a.ubuf, tcand = a.tcand;
+    fetch_U(sm.U, a.U, sm.cid, K, S);
+    cp_async_commit();
+    if (ubuf == 2) {
+      if (L > 1) fetch_U(sm.U + (size_t)K * S, a.U, sm.cid + K, K, S);
+      cp_async_commit();
+    }
     __syncthreads();
 
     int prev = x0, prank = 0;
+    float u_next = (a.select_mode == BRISK_SELECT_SAMPLE) ? a.u_sel[bL] : 0.f;
     for (int i = 0; i < L; ++i) {
       const int buf = i & 1;
       const int* ci = sm.cid + i * K;
+      // the token-share rows of the next position's previous token are among this position's
+      // candidates: stage them all (own chunks only) in shared memory, or pull them into L2
+      if (tcand) {
+        if (i + 1 < L) {
+          float* Tb = sm.Tc + (size_t)buf * K * 2 * S;
+          for (int k = 0; k < K; ++k) {
+            const float* src = a.Tzh + (size_t)ci[k] * 2 * S;
+#pragma unroll
+            for (int m = 0; m < MCH; ++m) {
+              const int c = tid + m * SCAN_THREADS;
+              if (c < nch) {
+                cp_async16(Tb + (size_t)k * 2 * S + 4 * c, src + 4 * c);
+                cp_async16(Tb + (size_t)k * 2 * S + S + 4 * c, src + S + 4 * c);
+              }
+            }
+          }
+        }
+        cp_async_commit();
+      } else if (i + 1 < L) {
+        prefetch_rows(a.Tzh, ci, K, 2 * S);
+      }
+      if (i + ubuf < L) prefetch_rows(a.U, ci + ubuf * K, K, S);
+      float* Ucur = sm.U + (size_t)(ubuf == 2 ? (i & 1) : 0) * K * S;
       // confidence features of position i (App. C.2)
       const float l0 = sm.top[i * 3 + 0];
       float phi[5];
@@ -406,38 +495,102 @@ scan_kernel(const __grid_constant__ ScanArgs a) {
       phi[2] = (prev == ci[0]) ? 1.f : 0.f;
       phi[3] = (prev == ci[0] || prev == ci[1] || prev == ci[2] || prev == ci[3]) ? 1.f : 0.f;
       phi[4] = l0 - sm.lprev[i * K + (i == 0 ? 0 : prank)];
-      // minimal-GRU step on this thread's state elements
-      const float* Gi = a.G + (bL + i) * 2 * S;
-      const float* Ti = a.Tzh + (size_t)prev * 2 * S;
+      // token share of the previous token (x0's was loaded in the prologue)
+      if (i > 0) {
+        if (tcand) {
+          const float* Tp = sm.Tc + ((size_t)((i - 1) & 1) * K + prank) * 2 * S;
+#pragma unroll
+          for (int m = 0; m < MCH; ++m) {
+            const int c = tid + m * SCAN_THREADS;
+            if (c < nch) {
+              tz4[m] = ld4(Tp + 4 * c);
+              th4[m] = ld4(Tp + S + 4 * c);
+            }
+          }
+        } else {
+          const float* Ti = a.Tzh + (size_t)prev * 2 * S;
+#pragma unroll
+          for (int m = 0; m < MCH; ++m) {
+            const int c = tid + m * SCAN_THREADS;
+            if (c < nch) {
+              tz4[m] = ld4(Ti + 4 * c);
+              th4[m] = ld4(Ti + S + 4 * c);
+            }
+          }
+        }
+      }
+      // minimal-GRU step on this thread's state chunks
       float gacc = 0.f;
 #pragma unroll
-      for (int q = 0; q < EPT_MAX; ++q) {
-        const int j = tid + q * SCAN_THREADS;
-        if (j < S) {
-          float zp = Gi[j] + a.posz[(size_t)i * S + j] + Ti[j];
-          float hp = Gi[S + j] + a.posh[(size_t)i * S + j] + Ti[S + j];
+      for (int m = 0; m < MCH; ++m) {
+        const int c = tid + m * SCAN_THREADS;
+        if (c < nch) {
+          float zp[4] = {gz4[m].x + tz4[m].x, gz4[m].y + tz4[m].y, gz4[m].z + tz4[m].z,
+                         gz4[m].w + tz4[m].w};
+          float hp[4] = {gh4[m].x + th4[m].x, gh4[m].y + th4[m].y, gh4[m].z + th4[m].z,
+                         gh4[m].w + th4[m].w};
 #pragma unroll
           for (int f = 0; f < 5; ++f) {
-            zp = fmaf(sm.F[f * S + j], phi[f], zp);
-            hp = fmaf(sm.F[(5 + f) * S + j], phi[f], hp);
+            const float4 fz = ld4(sm.F + (size_t)f * S + 4 * c);
+            const float4 fh = ld4(sm.F + (size_t)(5 + f) * S + 4 * c);
+            zp[0] = fmaf(fz.x, phi[f], zp[0]); zp[1] = fmaf(fz.y, phi[f], zp[1]);
+            zp[2] = fmaf(fz.z, phi[f], zp[2]); zp[3] = fmaf(fz.w, phi[f], zp[3]);
+            hp[0] = fmaf(fh.x, phi[f], hp[0]); hp[1] = fmaf(fh.y, phi[f], hp[1]);
+            hp[2] = fmaf(fh.z, phi[f], hp[2]); hp[3] = fmaf(fh.w, phi[f], hp[3]);
           }
-          const float z = sigmoidf_(zp);
-          s[q] = (1.f - z) * s[q] + z * hp;
-          sm.s[j] = s[q];
-          gacc = fmaf(wg[q], s[q], gacc);
+          float sv[4] = {s4[m].x, s4[m].y, s4[m].z, s4[m].w};
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            const float z = sigmoidf_(zp[e]);
+            sv[e] = (1.f - z) * sv[e] + z * hp[e];
+          }
+          s4[m] = make_float4(sv[0], sv[1], sv[2], sv[3]);
+          *reinterpret_cast<float4*>(sm.s + 4 * c) = s4[m];
+          gacc = fmaf(wg4[m].x, sv[0], gacc);
+          gacc = fmaf(wg4[m].y, sv[1], gacc);
+          gacc = fmaf(wg4[m].z, sv[2], gacc);
+          gacc = fmaf(wg4[m].w, sv[3], gacc);
+        }
+      }
+      // hidden and position shares of the next position: plain loads whose values are first
+      // used in the next step, so they stay in flight meanwhile
+      if (i + 1 < L) {
+        const float* Gn = a.G + (bL + i + 1) * 2 * S;
+#pragma unroll
+        for (int m = 0; m < MCH; ++m) {
+          const int c = tid + m * SCAN_THREADS;
+          if (c < nch) {
+            gz4[m] = ld4(Gn + 4 * c);
+            gh4[m] = ld4(Gn + S + 4 * c);
+          }
         }
       }
       gacc = warp_sum(gacc);
       if (lane == 0) sm.gpart[buf * SCAN_WARPS + warp] = gacc;
+      // this lane's residual rows of position i have landed (groups committed after them: the
+      // next position's rows, and this and the previous position's token-share batches)
+      if (tcand) cp_async_wait_pending(ubuf == 2 ? (i == 0 ? 2 : 3) : 1);
+      else cp_async_wait_pending(ubuf == 2 ? 1 : 0);
       __syncthreads();
-      // residual dots d_k = <s, U[c_k]>, one warp per candidate
+      // residual dots d_k = <s, U[c_k]>, one warp per candidate, rows from shared memory
       for (int k = warp; k < K; k += SCAN_WARPS) {
-        const float* Uc = a.U + (size_t)ci[k] * S;
+        const float4* Uk = reinterpret_cast<const float4*>(Ucur + (size_t)k * S);
+        const float4* s4 = reinterpret_cast<const float4*>(sm.s);
         float acc = 0.f;
-        for (int j = lane; j < S; j += 32) acc = fmaf(sm.s[j], Uc[j], acc);
+        for (int q = lane; q < S / 4; q += 32) {
+          const float4 u = Uk[q], v = s4[q];
+          acc = fmaf(u.x, v.x, acc);
+          acc = fmaf(u.y, v.y, acc);
+          acc = fmaf(u.z, v.z, acc);
+          acc = fmaf(u.w, v.w, acc);
+        }
         acc = warp_sum(acc);
         if (lane == 0) sm.d[buf * KMAX + k] = acc;
       }
+      // residual rows of position i + ubuf into the buffer just read (each lane refills exactly
+      // the chunks it read itself)
+      if (i + ubuf < L) fetch_U(Ucur, a.U, ci + ubuf * K, K, S);
+      cp_async_commit();
       __syncthreads();
       // gate, refined scores and Select (every thread, identical arithmetic)
       float gate = a.b_g;
@@ -445,14 +598,17 @@ scan_kernel(const __grid_constant__ ScanArgs a) {
 #pragma unroll
       for (int f = 0; f < 5; ++f) gate = fmaf(wgf[f], phi[f], gate);
       const float gamma = sig_alpha * sigmoidf_(gate);
-      float ref[KMAX];
-      for (int k = 0; k < K; ++k) ref[k] = sm.clp[i * K + k] + gamma * sm.d[buf * KMAX + k];
-      const float u = (a.select_mode == BRISK_SELECT_SAMPLE) ? a.u_sel[bL + i] : 0.f;
-      const int pick = select_rank(ref, K, a.select_mode, u);
+      const float* clp = sm.clp + i * K;
+      const float* dk = sm.d + buf * KMAX;
+      const int pick = select_rank(clp, dk, gamma, K, a.select_mode, u_next);
       if (tid < K) {
-        sm.ref[i * K + tid] = ref[tid];
-        a.refined[(bL + i) * K + tid] = ref[tid];
+        const float ref = clp[tid] + gamma * dk[tid];
+        sm.ref[i * K + tid] = ref;
+        a.refined[(bL + i) * K + tid] = ref;
       }
+      if (a.select_mode == BRISK_SELECT_SAMPLE && i + 1 < L) u_next = a.u_sel[bL + i + 1];
+      // this thread's token-share chunks of this position's candidates have landed
+      if (tcand) cp_async_wait_pending(1);
       prank = pick;
       prev = ci[pick];
       if (tid == 0) {
@@ -478,10 +634,33 @@ scan_kernel(const __grid_constant__ ScanArgs a) {
 
 }  // namespace
 
-size_t scan_smem_bytes(int L, int K, int S, int V) { return smem_layout(L, K, S, V, nullptr, nullptr); }
+constexpr size_t SCAN_SMEM_LIMIT = 227 * 1024;
 
-cudaError_t launch_scan(const ScanArgs& a, cudaStream_t stream) {
-  const size_t smem = scan_smem_bytes(a.L, a.K, a.S, a.V);
+// Shared-memory plan: double-buffered residual rows and staged token-share rows when they fit,
+// else fewer buffers.
+void scan_plan(int L, int K, int S, int V, int* ubuf, int* tcand) {
+  const int plans[3][2] = {{2, 1}, {2, 0}, {1, 0}};
+  for (const auto& p : plans) {
+    if (smem_layout(L, K, S, V, p[0], p[1], nullptr, nullptr) <= SCAN_SMEM_LIMIT) {
+      *ubuf = p[0];
+      *tcand = p[1];
+      return;
+    }
+  }
+  *ubuf = 1;
+  *tcand = 0;
+}
+
+size_t scan_smem_bytes(int L, int K, int S, int V) {
+  int ubuf, tcand;
+  scan_plan(L, K, S, V, &ubuf, &tcand);
+  return smem_layout(L, K, S, V, ubuf, tcand, nullptr, nullptr);
+}
+
+cudaError_t launch_scan(const ScanArgs& a_in, cudaStream_t stream) {
+  ScanArgs a = a_in;
+  scan_plan(a.L, a.K, a.S, a.V, &a.ubuf, &a.tcand);
+  const size_t smem = smem_layout(a.L, a.K, a.S, a.V, a.ubuf, a.tcand, nullptr, nullptr);
   cudaError_t e = cudaFuncSetAttribute(scan_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)smem);
   if (e != cudaSuccess) return e;

@@ -3,29 +3,31 @@
 // verifier rows the argmax (lowest id on ties) and the log-partition.
 //
 // Work unit: one warp sweeps one chunk of one row with coalesced 16-byte
-// streaming loads. Each lane keeps a running (max, sum of exp) pair and a
-// best-first list of KP >= K (logit, id) entries in registers; an element
-// costs one max, one exp and one add, and enters the list only when it beats
-// the list's last entry. The warp then merges its 32 lists and pairs. When a
-// row is split into several chunks, each warp writes its partial result to
-// the workspace and the last warp to finish the row (arrival counter)
-// merges the partials in chunk order, so results do not depend on timing.
+// streaming loads, SWEEP_UNROLL in flight per lane. Each lane keeps a running
+// (max, sum of exp) pair. The warp keeps one exact best-first list of the
+// chunk's top-K (logit, id) pairs spread over its lanes (lane k holds the
+// k-th best) and a warp-uniform threshold T, a lower bound on the K-th best
+// so far: a 16-byte vector whose max is below T cannot contribute, so the
+// common case costs one compare per vector. The rare vectors that reach T are
+// broadcast to the whole warp and their elements inserted cooperatively.
+// When a row is split into several chunks, each warp writes its partial
+// result to the workspace and the last warp to finish the row (arrival
+// counter, no waiting) merges the partials in chunk order, so results do not
+// depend on timing.
 #include "brisk_internal.cuh"
 
 namespace brisk {
 
 namespace {
 
-constexpr int SWEEP_WARPS = 4;            // independent warps per CTA
-constexpr int SWEEP_TARGET_TASKS = 152 * 48;  // warp tasks per tensor the chunking aims for
-constexpr int SWEEP_MIN_VEC_PER_LANE = 8;
+constexpr int SWEEP_WARPS = 4;                 // independent warps per CTA
+constexpr int SWEEP_UNROLL = 8;                // 16-byte loads in flight per lane
+constexpr int SWEEP_TARGET_TASKS = 152 * 24;   // warp tasks per tensor the chunking aims for
+constexpr int SWEEP_MIN_VEC_PER_LANE = 16;
 
-template <int KP, int N>
-__device__ __forceinline__ void consume(const float (&f)[N], int id0, float& m, float& s,
-                                        float (&vals)[KP], int (&ids)[KP]) {
-  float mx = f[0];
-#pragma unroll
-  for (int j = 1; j < N; ++j) mx = fmaxf(mx, f[j]);
+// Online log-sum-exp of one group of N logits whose max is mx.
+template <int N>
+__device__ __forceinline__ void lse_update(const float (&f)[N], float mx, float& m, float& s) {
   if (mx > m) {
     s *= ex2((m - mx) * LOG2E);
     m = mx;
@@ -40,10 +42,80 @@ __device__ __forceinline__ void consume(const float (&f)[N], int id0, float& m, 
     }
     s += a0 + a1;
   }
-  if (mx >= vals[KP - 1]) {
+}
+
+template <int N>
+__device__ __forceinline__ float max_of(const float (&f)[N]) {
+  float mx = f[0];
 #pragma unroll
-    for (int j = 0; j < N; ++j)
-      if (better(f[j], id0 + j, vals[KP - 1], ids[KP - 1])) list_insert<KP>(f[j], id0 + j, vals, ids);
+  for (int j = 1; j < N; ++j) mx = fmaxf(mx, f[j]);
+  return mx;
+}
+
+// Warp list: lane k < kout holds the k-th best (wv, wi); the other lanes hold (-inf, INVALID).
+// Cooperative insertion of (v, id), identical in every lane; returns the new K-th value.
+__device__ __forceinline__ float wlist_insert(float v, int id, float& wv, int& wi, int kout) {
+  const int lane = threadIdx.x & 31;
+  const bool ahead = lane < kout && !better(v, id, wv, wi);     // entries that stay before it
+  const int pos = __popc(__ballot_sync(FULL_MASK, ahead));
+  const float uv = __shfl_up_sync(FULL_MASK, wv, 1);
+  const int ui = __shfl_up_sync(FULL_MASK, wi, 1);
+  if (pos < kout && lane < kout) {
+    if (lane == pos) { wv = v; wi = id; }
+    else if (lane > pos) { wv = uv; wi = ui; }
+  }
+  return __shfl_sync(FULL_MASK, wv, kout - 1);
+}
+
+// k-th largest (k in 1..32) of one float per lane, the same in every lane (bitonic sort).
+__device__ __forceinline__ float warp_kth_largest(float x, int k) {
+  const int lane = threadIdx.x & 31;
+#pragma unroll
+  for (int size = 2; size <= 32; size <<= 1) {
+#pragma unroll
+    for (int j = size >> 1; j > 0; j >>= 1) {
+      const float y = __shfl_xor_sync(FULL_MASK, x, j);
+      const bool ascending = (lane & size) == 0;
+      const bool lower = (lane & j) == 0;
+      x = (lower == ascending) ? fminf(x, y) : fmaxf(x, y);
+    }
+  }
+  return __shfl_sync(FULL_MASK, x, 32 - k);
+}
+
+// Offer every element of the vector held by each lane in `trig` (a warp ballot) to the warp
+// list: the vector is broadcast, then its elements at or above T are inserted in id order.
+template <typename T>
+__device__ __forceinline__ void offer_vectors(unsigned trig, const uint4& w, int id0_lane,
+                                              float& thr, float& wv, int& wi, int kout) {
+  constexpr int VN = Vec<T>::N;
+  while (trig) {
+    const int src = __ffs(trig) - 1;
+    trig &= trig - 1;
+    uint4 b;
+    b.x = __shfl_sync(FULL_MASK, w.x, src);
+    b.y = __shfl_sync(FULL_MASK, w.y, src);
+    b.z = __shfl_sync(FULL_MASK, w.z, src);
+    b.w = __shfl_sync(FULL_MASK, w.w, src);
+    const int id0 = __shfl_sync(FULL_MASK, id0_lane, src);
+    float g[VN];
+    unpack(b, g, T());
+#pragma unroll
+    for (int j = 0; j < VN; ++j)
+      if (g[j] >= thr) thr = fmaxf(thr, wlist_insert(g[j], id0 + j, wv, wi, kout));
+  }
+}
+
+// One scalar element per lane (head or tail of a row), offered like a vector.
+__device__ __forceinline__ void offer_scalars(float f, int id, float& thr, float& wv, int& wi,
+                                              int kout) {
+  unsigned trig = __ballot_sync(FULL_MASK, f >= thr);
+  while (trig) {
+    const int src = __ffs(trig) - 1;
+    trig &= trig - 1;
+    const float g = __shfl_sync(FULL_MASK, f, src);
+    const int gid = __shfl_sync(FULL_MASK, id, src);
+    if (g >= thr) thr = fmaxf(thr, wlist_insert(g, gid, wv, wi, kout));
   }
 }
 
@@ -72,7 +144,7 @@ __device__ __forceinline__ void finalize_row(const SweepSeg& sg, int row, float 
   if (lane == 0) sg.out_lse[row] = lse;
 }
 
-template <typename T, int KP>
+template <typename T>
 __global__ void __launch_bounds__(SWEEP_WARPS * 32)
 sweep_kernel(const __grid_constant__ SweepLaunch a) {
   constexpr int VN = Vec<T>::N;
@@ -88,6 +160,7 @@ sweep_kernel(const __grid_constant__ SweepLaunch a) {
   const int row = (int)(t / a.nchunk);
   const int chunk = (int)(t % a.nchunk);
   const int V = a.V;
+  const int kout = sg.kout;
 
   const T* rowp = reinterpret_cast<const T*>(sg.logits) + (size_t)row * V;
   const uintptr_t addr = reinterpret_cast<uintptr_t>(rowp);
@@ -99,63 +172,81 @@ sweep_kernel(const __grid_constant__ SweepLaunch a) {
   const int v_begin = chunk * vpc;
   const int v_end = min(nvec, v_begin + vpc);
 
-  float m = -INFINITY, s = 0.f;
-  float vals[KP];
-  int ids[KP];
-  list_clear<KP>(vals, ids);
+  float m = -INFINITY, s = 0.f;        // this lane's running max and sum of exp(x - max)
+  float wv = -INFINITY;                // warp list entry held by this lane
+  int wi = INVALID_ID;
+  float thr = -INFINITY;               // warp-uniform lower bound on the K-th best so far
 
-  // unaligned head (ids below every vector): lane 0 of chunk 0
-  if (chunk == 0 && lane == 0) {
-    for (int e = 0; e < head; ++e) {
-      const float f[1] = {to_f32(rowp[e])};
-      consume<KP, 1>(f, e, m, s, vals, ids);
+  // unaligned head (ids below every vector): lanes 0..head-1 of chunk 0
+  if (chunk == 0) {
+    float f = -INFINITY;
+    if (lane < head) {
+      f = to_f32(rowp[lane]);
+      const float ff[1] = {f};
+      lse_update<1>(ff, f, m, s);
     }
+    offer_scalars(f, lane < head ? lane : INVALID_ID, thr, wv, wi, kout);
   }
   const uint4* vp = reinterpret_cast<const uint4*>(rowp + head);
-  int v = v_begin + lane;
-  for (; v + 96 < v_end; v += 128) {
-    const uint4 w0 = ld_stream_v4(vp + v);
-    const uint4 w1 = ld_stream_v4(vp + v + 32);
-    const uint4 w2 = ld_stream_v4(vp + v + 64);
-    const uint4 w3 = ld_stream_v4(vp + v + 96);
-    float f[VN];
-    unpack(w0, f, T());
-    consume<KP, VN>(f, head + v * VN, m, s, vals, ids);
-    unpack(w1, f, T());
-    consume<KP, VN>(f, head + (v + 32) * VN, m, s, vals, ids);
-    unpack(w2, f, T());
-    consume<KP, VN>(f, head + (v + 64) * VN, m, s, vals, ids);
-    unpack(w3, f, T());
-    consume<KP, VN>(f, head + (v + 96) * VN, m, s, vals, ids);
+  bool first = true;
+  for (int base = v_begin; base < v_end; base += 32 * SWEEP_UNROLL) {
+    uint4 w[SWEEP_UNROLL];
+#pragma unroll
+    for (int u = 0; u < SWEEP_UNROLL; ++u) {
+      const int v = base + lane + 32 * u;
+      if (v < v_end) w[u] = ld_stream_v4(vp + v);
+      else w[u] = make_uint4(0xff80ff80u, 0xff80ff80u, 0xff80ff80u, 0xff80ff80u);  // -inf
+    }
+    if constexpr (VN == 4) {
+#pragma unroll
+      for (int u = 0; u < SWEEP_UNROLL; ++u)
+        if (base + lane + 32 * u >= v_end) w[u] = make_uint4(0xff800000u, 0xff800000u, 0xff800000u, 0xff800000u);
+    }
+    float mx[SWEEP_UNROLL];
+    float mx_all = -INFINITY;
+#pragma unroll
+    for (int u = 0; u < SWEEP_UNROLL; ++u) {
+      float f[VN];
+      unpack(w[u], f, T());
+      mx[u] = max_of(f);
+      lse_update<VN>(f, mx[u], m, s);
+      mx_all = fmaxf(mx_all, mx[u]);
+    }
+    if (first) {
+      // K lanes each hold an element at least this large: a lower bound on the K-th best
+      thr = fmaxf(thr, warp_kth_largest(mx_all, kout));
+      first = false;
+    }
+#pragma unroll
+    for (int u = 0; u < SWEEP_UNROLL; ++u) {
+      const unsigned trig = __ballot_sync(FULL_MASK, mx[u] >= thr);
+      if (trig) offer_vectors<T>(trig, w[u], head + (base + lane + 32 * u) * VN, thr, wv, wi, kout);
+    }
   }
-  for (; v < v_end; v += 32) {
-    const uint4 w0 = ld_stream_v4(vp + v);
-    float f[VN];
-    unpack(w0, f, T());
-    consume<KP, VN>(f, head + v * VN, m, s, vals, ids);
-  }
-  // ragged tail (ids above every vector): last chunk, one element per lane
+  // ragged tail (ids above every vector): lanes of the last chunk, one element each
   if (chunk == a.nchunk - 1) {
     const int e = tail0 + lane;
+    float f = -INFINITY;
     if (e < V) {
-      const float f[1] = {to_f32(rowp[e])};
-      consume<KP, 1>(f, e, m, s, vals, ids);
+      f = to_f32(rowp[e]);
+      const float ff[1] = {f};
+      lse_update<1>(ff, f, m, s);
     }
+    offer_scalars(f, e < V ? e : INVALID_ID, thr, wv, wi, kout);
   }
 
   warp_lse_combine(m, s);
-  float ov;
-  int oi;
-  warp_extract<KP>(vals, ids, sg.kout, ov, oi);
+  const float ov = wv;
+  const int oi = wi;
   if (a.nchunk == 1) {
     finalize_row(sg, row, m, s, ov, oi, a.status);
     return;
   }
 
   const size_t pb = (size_t)row * a.nchunk + chunk;
-  if (lane < sg.kout) {
-    sg.part_val[pb * KP + lane] = ov;
-    sg.part_id[pb * KP + lane] = oi;
+  if (lane < kout) {
+    sg.part_val[pb * a.KP + lane] = ov;
+    sg.part_id[pb * a.KP + lane] = oi;
   }
   if (lane == 0) {
     sg.part_m[pb] = m;
@@ -170,12 +261,18 @@ sweep_kernel(const __grid_constant__ SweepLaunch a) {
   __threadfence();
 
   // last warp of the row: merge the chunk partials in chunk order
-  list_clear<KP>(vals, ids);
-  const int nent = a.nchunk * sg.kout;
-  for (int e = lane; e < nent; e += 32) {
-    const int c = e / sg.kout, k = e - c * sg.kout;
-    const size_t q = ((size_t)row * a.nchunk + c) * KP + k;
-    list_insert<KP>(__ldcg(sg.part_val + q), __ldcg(sg.part_id + q), vals, ids);
+  wv = -INFINITY;
+  wi = INVALID_ID;
+  thr = -INFINITY;
+  for (int c = 0; c < a.nchunk; ++c) {
+    const size_t q = ((size_t)row * a.nchunk + c) * a.KP;
+    float f = -INFINITY;
+    int id = INVALID_ID;
+    if (lane < kout) {
+      f = __ldcg(sg.part_val + q + lane);
+      id = __ldcg(sg.part_id + q + lane);
+    }
+    offer_scalars(f, id, thr, wv, wi, kout);
   }
   float mm = -INFINITY, ss = 0.f;
   for (int c = lane; c < a.nchunk; c += 32) {
@@ -183,8 +280,7 @@ sweep_kernel(const __grid_constant__ SweepLaunch a) {
     lse_merge(mm, ss, __ldcg(sg.part_m + q), __ldcg(sg.part_s + q));
   }
   warp_lse_combine(mm, ss);
-  warp_extract<KP>(vals, ids, sg.kout, ov, oi);
-  finalize_row(sg, row, mm, ss, ov, oi, a.status);
+  finalize_row(sg, row, mm, ss, wv, wi, a.status);
   if (lane == 0) sg.counters[row] = 0;
 }
 
@@ -193,14 +289,7 @@ cudaError_t launch_t(const SweepLaunch& a, cudaStream_t stream) {
   long long tasks = (long long)a.seg[0].rows * a.nchunk;
   if (a.nseg > 1) tasks += (long long)a.seg[1].rows * a.nchunk;
   const unsigned grid = (unsigned)((tasks + SWEEP_WARPS - 1) / SWEEP_WARPS);
-  const dim3 block(SWEEP_WARPS * 32);
-  switch (a.KP) {
-    case 4: sweep_kernel<T, 4><<<grid, block, 0, stream>>>(a); break;
-    case 8: sweep_kernel<T, 8><<<grid, block, 0, stream>>>(a); break;
-    case 16: sweep_kernel<T, 16><<<grid, block, 0, stream>>>(a); break;
-    case 32: sweep_kernel<T, 32><<<grid, block, 0, stream>>>(a); break;
-    default: return cudaErrorInvalidValue;
-  }
+  sweep_kernel<T><<<grid, SWEEP_WARPS * 32, 0, stream>>>(a);
   return cudaGetLastError();
 }
 
