@@ -44,7 +44,8 @@ class TailIO(ctypes.Structure):
 
 
 class Events(ctypes.Structure):
-    _fields_ = [("sweep_begin", _vp), ("sweep_end", _vp)]
+    _fields_ = [("sweep_q_begin", _vp), ("sweep_q_end", _vp), ("sweep_p_begin", _vp),
+                ("sweep_p_end", _vp)]
 
 
 class BriskError(RuntimeError):
@@ -239,7 +240,7 @@ class DecodeTail:
                     _p(out["correction"]), _p(out.get("next_anchor")))
         ev = None
         if events is not None:
-            ev = ctypes.byref(Events(_vp(events[0].cuda_event), _vp(events[1].cuda_event)))
+            ev = ctypes.byref(Events(*[_vp(e.cuda_event) for e in events]))
         _check(lib().brisk_decode_tail(ctypes.byref(self.dims), ctypes.byref(self.params),
                                        _p(self.tables), ctypes.byref(io), int(select_mode),
                                        int(verify_mode), _p(self.workspace), ev, _stream(stream)),

@@ -1,4 +1,5 @@
 // C ABI of the decode tail: argument checks, workspace and table layouts, launches.
+#include <mutex>
 #include <string.h>
 
 #include "brisk_internal.cuh"
@@ -148,7 +149,7 @@ SweepSeg make_seg(const WsLayout& w, void* ws, int seg, const void* logits, int 
 // second one multiplies by the weight blocks written three times along k (fp32-level accuracy).
 brisk_status hidden_products(const brisk_dims* d, const brisk_params* p, const void* tables,
                              const void* hidden, const void* h_ctx, const WsLayout& w, void* ws,
-                             cudaStream_t st) {
+                             cudaStream_t st, int stages = 4) {
   const TbLayout t = tb_layout(d);
   const int BL = d->B * d->L, r = d->r, S = 2 * d->r, hd = d->hidden_dtype;
   int32_t* status = at<int32_t>(ws, w.status);
@@ -159,13 +160,13 @@ brisk_status hidden_products(const brisk_dims* d, const brisk_params* p, const v
     const TcSpec first[2] = {
         {BL, r, d->d, hidden, d->d, p->P_h, d->d, 1, Hs, r3, nullptr, 0},
         {d->B, r, d->d, h_ctx, d->d, p->P_h, d->d, 1, Hs + (size_t)BL * r3, r3, nullptr, 0}};
-    BRISK_CUDA(gemm_tc_grouped(first, 2, status, st));
+    BRISK_CUDA(gemm_tc_grouped(first, 2, status, st, stages));
     const TcSpec second[2] = {
         {BL, 2 * S, r3, Hs, r3, at<__nv_bfloat16>(tables, t.W2s), r3, 0, at<float>(ws, w.G), 2 * S,
          at<float>(tables, t.posG), d->L},
         {d->B, S, r3, Hs + (size_t)BL * r3, r3, at<__nv_bfloat16>(tables, t.W0s), r3, 0,
          at<float>(ws, w.G0), S, nullptr, 0}};
-    BRISK_CUDA(gemm_tc_grouped(second, 2, status, st));
+    BRISK_CUDA(gemm_tc_grouped(second, 2, status, st, stages));
     return BRISK_OK;
   }
   float* Hm = at<float>(ws, w.Hm);
@@ -177,6 +178,30 @@ brisk_status hidden_products(const brisk_dims* d, const brisk_params* p, const v
   BRISK_CUDA(gemm_simt(d->B, S, r, Hm + (size_t)BL * r, BRISK_DT_F32, r, at<float>(tables, t.W0h),
                        BRISK_DT_F32, r, false, at<float>(ws, w.G0), S, st));
   return BRISK_OK;
+}
+
+// A side stream per device (created on the first fused call on that device) and the events that
+// fork work onto it and join it back, so that one call can run independent stages concurrently.
+struct SideStream {
+  cudaStream_t stream = nullptr;
+  cudaEvent_t ev[3] = {nullptr, nullptr, nullptr};
+};
+constexpr int MAX_DEVICES = 256;
+std::mutex g_side_mu;
+SideStream g_side[MAX_DEVICES];
+
+SideStream* side_stream() {
+  int dev = -1;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= MAX_DEVICES) return nullptr;
+  SideStream& ss = g_side[dev];
+  if (!ss.stream) {
+    cudaStream_t st = nullptr;
+    if (cudaStreamCreateWithFlags(&st, cudaStreamNonBlocking) != cudaSuccess) return nullptr;
+    for (auto& e : ss.ev)
+      if (cudaEventCreateWithFlags(&e, cudaEventDisableTiming) != cudaSuccess) return nullptr;
+    ss.stream = st;
+  }
+  return &ss;
 }
 
 ScanArgs scan_args(const brisk_dims* d, const brisk_params* p, const void* tables, const WsLayout& w,
@@ -410,27 +435,42 @@ brisk_status brisk_decode_tail(const brisk_dims* d, const brisk_params* p, const
   int32_t* sel = io->sel_tokens ? io->sel_tokens : at<int32_t>(ws, w.sel);
   float* refined = io->refined ? io->refined : at<float>(ws, w.refined);
 
-  SweepLaunch sw{};
-  sw.seg[0] = make_seg(w, ws, 0, io->logits_q, BL, d->K, cand_ids, cand_lp, lse_q);
-  sw.seg[1] = make_seg(w, ws, 1, io->logits_p, BL, 1, at<int32_t>(ws, w.argmax_p), nullptr,
-                       at<float>(ws, w.lse_p));
-  sw.nseg = 2;
-  sw.V = d->V;
-  sw.nchunk = w.nchunk;
-  sw.KP = w.KP;
-  sw.dtype = d->logits_dtype;
-  sw.status = at<int32_t>(ws, w.status);
-  if (ev && ev->sweep_begin) BRISK_CUDA(cudaEventRecord(static_cast<cudaEvent_t>(ev->sweep_begin), st));
-  BRISK_CUDA(launch_sweep(sw, st));
-  if (ev && ev->sweep_end) BRISK_CUDA(cudaEventRecord(static_cast<cudaEvent_t>(ev->sweep_end), st));
-
-  s = hidden_products(d, p, tables, io->hidden, io->h_ctx, w, ws, st);
+  // Schedule (A = caller's stream, B = side stream):
+  //   A: proposal-row sweep ............ verifier-row sweep ... join ... verification
+  //   B: hidden-state products ... join ... corrector scan
+  // The corrector needs only the proposal candidates and the hidden products; the verifier rows
+  // are needed only by the verification, so the corrector runs under the second sweep.
+  std::lock_guard<std::mutex> lock(g_side_mu);
+  SideStream* ss = side_stream();
+  if (!ss) return BRISK_ERR_CUDA;
+  cudaStream_t sb = ss->stream;
+  BRISK_CUDA(cudaEventRecord(ss->ev[0], st));
+  BRISK_CUDA(cudaStreamWaitEvent(sb, ss->ev[0], 0));
+  s = hidden_products(d, p, tables, io->hidden, io->h_ctx, w, ws, sb, 2);
   if (s != BRISK_OK) return s;
+
+  SweepLaunch sq{};
+  sq.seg[0] = make_seg(w, ws, 0, io->logits_q, BL, d->K, cand_ids, cand_lp, lse_q);
+  sq.nseg = 1;
+  sq.V = d->V;
+  sq.nchunk = w.nchunk;
+  sq.KP = w.KP;
+  sq.dtype = d->logits_dtype;
+  sq.status = at<int32_t>(ws, w.status);
+  SweepLaunch sp = sq;
+  sp.seg[0] = make_seg(w, ws, 1, io->logits_p, BL, 1, at<int32_t>(ws, w.argmax_p), nullptr,
+                       at<float>(ws, w.lse_p));
+  if (ev && ev->sweep_q_begin) BRISK_CUDA(cudaEventRecord(static_cast<cudaEvent_t>(ev->sweep_q_begin), st));
+  BRISK_CUDA(launch_sweep(sq, st));
+  if (ev && ev->sweep_q_end) BRISK_CUDA(cudaEventRecord(static_cast<cudaEvent_t>(ev->sweep_q_end), st));
+  BRISK_CUDA(cudaEventRecord(ss->ev[1], st));
+
+  BRISK_CUDA(cudaStreamWaitEvent(sb, ss->ev[1], 0));
   ScanArgs a = scan_args(d, p, tables, w, ws);
   a.select_mode = select_mode;
   a.verify_mode = verify_mode;
   a.do_select = 1;
-  a.do_verify = 1;
+  a.do_verify = 0;
   a.logits_q = io->logits_q;
   a.cand_ids = cand_ids;
   a.cand_logprob = cand_lp;
@@ -438,21 +478,38 @@ brisk_status brisk_decode_tail(const brisk_dims* d, const brisk_params* p, const
   a.u_sel = io->u_sel;
   a.sel_tokens = sel;
   a.refined = refined;
-  a.logits_p = io->logits_p;
-  a.u_acc = io->u_acc;
-  a.u_res = io->u_res;
-  a.accepted_len = io->accepted_len;
-  a.out_tokens = io->out_tokens;
-  a.correction = io->correction;
-  a.next_anchor = io->next_anchor;
-  BRISK_CUDA(launch_scan(a, st));
+  BRISK_CUDA(launch_scan(a, sb));
+  BRISK_CUDA(cudaEventRecord(ss->ev[2], sb));
+
+  if (ev && ev->sweep_p_begin) BRISK_CUDA(cudaEventRecord(static_cast<cudaEvent_t>(ev->sweep_p_begin), st));
+  BRISK_CUDA(launch_sweep(sp, st));
+  if (ev && ev->sweep_p_end) BRISK_CUDA(cudaEventRecord(static_cast<cudaEvent_t>(ev->sweep_p_end), st));
+  BRISK_CUDA(cudaStreamWaitEvent(st, ss->ev[2], 0));
+
+  ScanArgs v = scan_args(d, nullptr, nullptr, w, ws);
+  v.select_mode = select_mode;
+  v.verify_mode = verify_mode;
+  v.do_select = 0;
+  v.do_verify = 1;
+  v.cand_ids = cand_ids;
+  v.sel_tokens = sel;
+  v.refined = refined;
+  v.logits_p = io->logits_p;
+  v.u_acc = io->u_acc;
+  v.u_res = io->u_res;
+  v.accepted_len = io->accepted_len;
+  v.out_tokens = io->out_tokens;
+  v.correction = io->correction;
+  v.next_anchor = io->next_anchor;
+  BRISK_CUDA(launch_scan(v, st));
   return BRISK_OK;
 }
 
 int32_t brisk_kernels_per_tail(const brisk_dims* dims) {
   if (!dims_ok(dims)) return 0;
   const bool tc = dims->hidden_dtype == BRISK_DT_BF16;
-  return 1 /* sweep */ + (tc ? 2 : 4) /* hidden-state products */ + 1 /* scan + verify */;
+  // two sweeps, the hidden-state products, the corrector scan, the verification
+  return 2 + (tc ? 2 : 4) + 1 + 1;
 }
 
 brisk_status brisk_last_device_status(void* ws, int32_t clear, void* stream) {

@@ -199,7 +199,10 @@ struct TcSpec {
   const float* bias;   // optional fp32 [bias_period, N] added to row m as bias[m % bias_period] (mode 0)
   int bias_period;
 };
-cudaError_t gemm_tc_grouped(const TcSpec* spec, int nprob, int32_t* status, cudaStream_t stream);
+// `stages` (2 or 4) sets the shared-memory pipeline depth: 2 leaves room on each SM for other
+// kernels running concurrently.
+cudaError_t gemm_tc_grouped(const TcSpec* spec, int nprob, int32_t* status, cudaStream_t stream,
+                            int stages);
 bool gemm_tc_supported(const void* A, int lda, const void* B, int ldb, int K);
 // dst[i*ldd + j] = (dst type) src[i*lds + j], i < rows, j < cols.
 cudaError_t copy2d(int rows, int cols, const void* src, int s_dt, int lds, void* dst, int d_dt,

@@ -25,7 +25,7 @@ namespace {
 
 constexpr int TC_BM = 128;
 constexpr int TC_BK = 64;               // one 128-byte swizzle row of bf16
-constexpr int TC_STAGES = 4;
+constexpr int TC_STAGES_MAX = 4;
 constexpr int TC_THREADS = 128;
 constexpr long long WAIT_LIMIT_CYCLES = 4000000000ll;   // about 2 s of SM clock per wait
 
@@ -157,6 +157,7 @@ struct TcArgs {
   int32_t* status;
 };
 
+template <int TC_STAGES>
 __global__ void __launch_bounds__(TC_THREADS, 1)
 gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__ CUtensorMap tmB0,
                const __grid_constant__ CUtensorMap tmA1, const __grid_constant__ CUtensorMap tmB1,
@@ -246,48 +247,64 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__
   }
   __syncthreads();
   tc_fence_after();
-  // Every warp owns TMEM lanes [32*warp, 32*warp + 32) = tile rows. Each 32 x 32 block goes
-  // through a padded shared-memory tile (the stage buffers are idle now) so that the global
-  // stores run along rows: one coalesced row segment per store instruction.
+  // Every warp owns TMEM lanes [32*warp, 32*warp + 32) = tile rows: each thread holds one row
+  // and writes it 32 columns at a time with 16-byte stores (a row segment per thread).
   if (!*abort_flag) {
-    float* stage = reinterpret_cast<float*>(base) + warp * (32 * 33);
     const uint32_t trow = tmem + (static_cast<uint32_t>(warp * 32) << 16);
-    const int row0 = m0 + warp * 32;
+    const int row = m0 + warp * 32 + lane;
+    const bool live = row < P.M;
+    const float* brow = (P.bias && live) ? P.bias + (size_t)(row % P.bias_period) * P.N : nullptr;
     for (int c0 = 0; c0 < a.BN; c0 += 32) {
       float v[32];
       tmem_ld32(trow + c0, v);
+      const int nb = n0 + c0;
+      if (!live || nb >= P.N) continue;
+      if (P.mode == 0) {
+        float* Cr = static_cast<float*>(P.C) + (size_t)row * P.ldc + nb;
+        if (brow) {
 #pragma unroll
-      for (int j = 0; j < 32; ++j) stage[lane * 33 + j] = v[j];
-      __syncwarp();
-      const int n = n0 + c0 + lane;
-      if (n < P.N) {
-        if (P.mode == 0) {
-          float* C = static_cast<float*>(P.C);
-          float bias[32];
+          for (int q = 0; q < 8; ++q)
+            if (nb + 4 * q + 3 < P.N) {
+              const float4 b = __ldg(reinterpret_cast<const float4*>(brow + nb) + q);
+              v[4 * q] += b.x; v[4 * q + 1] += b.y; v[4 * q + 2] += b.z; v[4 * q + 3] += b.w;
+            }
+        }
 #pragma unroll
-          for (int rr = 0; rr < 32; ++rr)   // independent loads, all in flight before the stores
-            bias[rr] = (P.bias && row0 + rr < P.M)
-                           ? __ldg(P.bias + (size_t)((row0 + rr) % P.bias_period) * P.N + n)
-                           : 0.f;
+        for (int q = 0; q < 8; ++q) {
+          if (nb + 4 * q + 3 < P.N) {
+            reinterpret_cast<float4*>(Cr)[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+          } else {
+            for (int e = 0; e < 4; ++e)
+              if (nb + 4 * q + e < P.N) Cr[4 * q + e] = v[4 * q + e] + (brow ? brow[nb + 4 * q + e] : 0.f);
+          }
+        }
+      } else {
+        // three bf16 parts, hi + mid + lo = x to about 2^-24 relative
+        __nv_bfloat16* Cr = static_cast<__nv_bfloat16*>(P.C) + (size_t)row * P.ldc + nb;
+        __align__(16) __nv_bfloat16 hi[32], mid[32], lo[32];
 #pragma unroll
-          for (int rr = 0; rr < 32; ++rr)
-            if (row0 + rr < P.M) C[(size_t)(row0 + rr) * P.ldc + n] = stage[rr * 33 + lane] + bias[rr];
-        } else {
-          __nv_bfloat16* C = static_cast<__nv_bfloat16*>(P.C);
-          for (int rr = 0; rr < 32 && row0 + rr < P.M; ++rr) {
-            // three bf16 parts, hi + mid + lo = x to about 2^-24 relative
-            const float x = stage[rr * 33 + lane];
-            const __nv_bfloat16 hi = __float2bfloat16_rn(x);
-            const float r1 = x - __bfloat162float(hi);
-            const __nv_bfloat16 mid = __float2bfloat16_rn(r1);
-            __nv_bfloat16* Cr = C + (size_t)(row0 + rr) * P.ldc;
-            Cr[n] = hi;
-            Cr[P.N + n] = mid;
-            Cr[2 * P.N + n] = __float2bfloat16_rn(r1 - __bfloat162float(mid));
+        for (int j = 0; j < 32; ++j) {
+          hi[j] = __float2bfloat16_rn(v[j]);
+          const float r1 = v[j] - __bfloat162float(hi[j]);
+          mid[j] = __float2bfloat16_rn(r1);
+          lo[j] = __float2bfloat16_rn(r1 - __bfloat162float(mid[j]));
+        }
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          if (nb + 8 * q + 7 < P.N) {
+            reinterpret_cast<uint4*>(Cr)[q] = reinterpret_cast<const uint4*>(hi)[q];
+            reinterpret_cast<uint4*>(Cr + P.N)[q] = reinterpret_cast<const uint4*>(mid)[q];
+            reinterpret_cast<uint4*>(Cr + 2 * P.N)[q] = reinterpret_cast<const uint4*>(lo)[q];
+          } else {
+            for (int e = 0; e < 8; ++e)
+              if (nb + 8 * q + e < P.N) {
+                Cr[8 * q + e] = hi[8 * q + e];
+                Cr[P.N + 8 * q + e] = mid[8 * q + e];
+                Cr[2 * P.N + 8 * q + e] = lo[8 * q + e];
+              }
           }
         }
       }
-      __syncwarp();
     }
   } else if (lane == 0) {
     set_status(a.status, BRISK_ERR_TIMEOUT);
@@ -335,8 +352,8 @@ bool make_map(CUtensorMap* map, const void* ptr, int rows, int cols, int ld, int
 
 }  // namespace
 
-size_t gemm_tc_smem(int BN) {
-  return 1024 + TC_STAGES * (TC_BM * TC_BK * 2 + BN * TC_BK * 2) + (2 * TC_STAGES + 1) * 8 + 16;
+size_t gemm_tc_smem(int BN, int stages) {
+  return 1024 + stages * (TC_BM * TC_BK * 2 + BN * TC_BK * 2) + (2 * TC_STAGES_MAX + 1) * 8 + 16;
 }
 
 bool gemm_tc_supported(const void* A, int lda, const void* B, int ldb, int K) {
@@ -346,8 +363,9 @@ bool gemm_tc_supported(const void* A, int lda, const void* B, int ldb, int K) {
 
 // One or two products C = A B^T, A [M, K] (row stride lda) and B [N, K] (row stride ldb) bf16,
 // fp32 accumulation, in one launch.
-cudaError_t gemm_tc_grouped(const TcSpec* spec, int nprob, int32_t* status, cudaStream_t stream) {
-  if (nprob < 1 || nprob > 2) return cudaErrorInvalidValue;
+cudaError_t gemm_tc_grouped(const TcSpec* spec, int nprob, int32_t* status, cudaStream_t stream,
+                            int stages) {
+  if (nprob < 1 || nprob > 2 || (stages != 2 && stages != 4)) return cudaErrorInvalidValue;
   int nmax = 0;
   for (int i = 0; i < nprob; ++i) nmax = spec[i].N > nmax ? spec[i].N : nmax;
   int BN = ((nmax + 15) / 16) * 16;
@@ -377,11 +395,18 @@ cudaError_t gemm_tc_grouped(const TcSpec* spec, int nprob, int32_t* status, cuda
     total += P.mtiles * P.ntiles;
   }
   if (total == 0) return cudaSuccess;
-  const size_t smem = gemm_tc_smem(BN);
-  cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       static_cast<int>(smem));
-  if (e != cudaSuccess) return e;
-  gemm_tc_kernel<<<total, TC_THREADS, smem, stream>>>(maps[0], maps[1], maps[2], maps[3], a);
+  const size_t smem = gemm_tc_smem(BN, stages);
+  if (stages == 2) {
+    cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
+    gemm_tc_kernel<2><<<total, TC_THREADS, smem, stream>>>(maps[0], maps[1], maps[2], maps[3], a);
+  } else {
+    cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
+    gemm_tc_kernel<4><<<total, TC_THREADS, smem, stream>>>(maps[0], maps[1], maps[2], maps[3], a);
+  }
   return cudaGetLastError();
 }
 
@@ -389,7 +414,7 @@ cudaError_t gemm_tc(int M, int N, int K, const void* A, int lda, const void* B, 
                     void* C, int ldc, int32_t* status, cudaStream_t stream) {
   if (M <= 0 || N <= 0) return cudaSuccess;
   const TcSpec s{M, N, K, A, lda, B, ldb, mode, C, ldc, nullptr, 0};
-  return gemm_tc_grouped(&s, 1, status, stream);
+  return gemm_tc_grouped(&s, 1, status, stream, 4);
 }
 
 }  // namespace brisk

@@ -22,8 +22,8 @@ namespace {
 
 constexpr int SWEEP_WARPS = 4;                 // independent warps per CTA
 constexpr int SWEEP_UNROLL = 8;                // 16-byte loads in flight per lane
-constexpr int SWEEP_TARGET_TASKS = 152 * 24;   // warp tasks per tensor the chunking aims for
-constexpr int SWEEP_MIN_VEC_PER_LANE = 16;
+constexpr int SWEEP_TARGET_TASKS = 152 * 16;   // warp tasks per tensor the chunking aims for
+constexpr int SWEEP_MIN_VEC_PER_LANE = 32;
 
 // Online log-sum-exp of one group of N logits whose max is mx.
 template <int N>
@@ -83,26 +83,38 @@ __device__ __forceinline__ float warp_kth_largest(float x, int k) {
   return __shfl_sync(FULL_MASK, x, 32 - k);
 }
 
-// Offer every element of the vector held by each lane in `trig` (a warp ballot) to the warp
-// list: the vector is broadcast, then its elements at or above T are inserted in id order.
+// The rare path. Every lane of the warp has stashed its SWEEP_UNROLL vectors in shared memory;
+// vector u of lane l holds ids id0(l) + u * 32 * VN + j. Each vector whose max reaches T is read
+// by the whole warp (a broadcast from shared memory) and its elements at or above T are
+// inserted in id order. Kept out of the unrolled main loop: one copy of the insertion code.
 template <typename T>
-__device__ __forceinline__ void offer_vectors(unsigned trig, const uint4& w, int id0_lane,
-                                              float& thr, float& wv, int& wi, int kout) {
+__device__ __forceinline__ void offer_stash(const uint4* warp_stash, unsigned umask, int id0_lane,
+                                         float& thr, float& wv, int& wi, int kout) {
   constexpr int VN = Vec<T>::N;
-  while (trig) {
-    const int src = __ffs(trig) - 1;
-    trig &= trig - 1;
-    uint4 b;
-    b.x = __shfl_sync(FULL_MASK, w.x, src);
-    b.y = __shfl_sync(FULL_MASK, w.y, src);
-    b.z = __shfl_sync(FULL_MASK, w.z, src);
-    b.w = __shfl_sync(FULL_MASK, w.w, src);
-    const int id0 = __shfl_sync(FULL_MASK, id0_lane, src);
-    float g[VN];
-    unpack(b, g, T());
-#pragma unroll
-    for (int j = 0; j < VN; ++j)
-      if (g[j] >= thr) thr = fmaxf(thr, wlist_insert(g[j], id0 + j, wv, wi, kout));
+  const int lane = threadIdx.x & 31;
+#pragma unroll 1
+  while (umask) {   // only the vector slots u where some lane reached the threshold
+    const int u = __ffs(umask) - 1;
+    umask &= umask - 1;
+    float f[VN];
+    unpack(warp_stash[lane * SWEEP_UNROLL + u], f, T());
+    unsigned trig = __ballot_sync(FULL_MASK, max_of(f) >= thr);
+    while (trig) {
+      const int src = __ffs(trig) - 1;
+      trig &= trig - 1;
+      // lane j < VN reads element j of lane src's vector; the ones at or above T are inserted
+      // in id order
+      const T* e = reinterpret_cast<const T*>(warp_stash + src * SWEEP_UNROLL + u);
+      const float g = lane < VN ? to_f32(e[lane]) : -INFINITY;
+      const int id0 = __shfl_sync(FULL_MASK, id0_lane, src) + u * 32 * VN;
+      unsigned em = __ballot_sync(FULL_MASK, lane < VN && g >= thr);
+      while (em) {
+        const int j = __ffs(em) - 1;
+        em &= em - 1;
+        const float gj = __shfl_sync(FULL_MASK, g, j);
+        if (gj >= thr) thr = fmaxf(thr, wlist_insert(gj, id0 + j, wv, wi, kout));
+      }
+    }
   }
 }
 
@@ -148,8 +160,10 @@ template <typename T>
 __global__ void __launch_bounds__(SWEEP_WARPS * 32)
 sweep_kernel(const __grid_constant__ SweepLaunch a) {
   constexpr int VN = Vec<T>::N;
+  __shared__ uint4 stash[SWEEP_WARPS * 32 * SWEEP_UNROLL];
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
+  uint4* warp_stash = stash + warp * 32 * SWEEP_UNROLL;
   const long long task = (long long)blockIdx.x * SWEEP_WARPS + warp;
   const long long tasks0 = (long long)a.seg[0].rows * a.nchunk;
   const long long total = tasks0 + (a.nseg > 1 ? (long long)a.seg[1].rows * a.nchunk : 0);
@@ -217,10 +231,16 @@ sweep_kernel(const __grid_constant__ SweepLaunch a) {
       thr = fmaxf(thr, warp_kth_largest(mx_all, kout));
       first = false;
     }
+    unsigned umask = 0;
 #pragma unroll
-    for (int u = 0; u < SWEEP_UNROLL; ++u) {
-      const unsigned trig = __ballot_sync(FULL_MASK, mx[u] >= thr);
-      if (trig) offer_vectors<T>(trig, w[u], head + (base + lane + 32 * u) * VN, thr, wv, wi, kout);
+    for (int u = 0; u < SWEEP_UNROLL; ++u) umask |= (mx[u] >= thr ? 1u : 0u) << u;
+    umask = __reduce_or_sync(FULL_MASK, umask);
+    if (umask) {
+#pragma unroll
+      for (int u = 0; u < SWEEP_UNROLL; ++u) warp_stash[lane * SWEEP_UNROLL + u] = w[u];
+      __syncwarp();
+      offer_stash<T>(warp_stash, umask, head + (base + lane) * VN, thr, wv, wi, kout);
+      __syncwarp();
     }
   }
   // ragged tail (ids above every vector): lanes of the last chunk, one element each
