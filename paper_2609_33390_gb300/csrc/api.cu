@@ -195,8 +195,13 @@ SideStream* side_stream() {
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= MAX_DEVICES) return nullptr;
   SideStream& ss = g_side[dev];
   if (!ss.stream) {
+    // highest priority: when a stage on the side stream becomes ready together with a sweep on
+    // the caller's stream, its blocks are placed first and the sweep fills the remaining room
+    int least = 0, greatest = 0;
+    if (cudaDeviceGetStreamPriorityRange(&least, &greatest) != cudaSuccess) return nullptr;
     cudaStream_t st = nullptr;
-    if (cudaStreamCreateWithFlags(&st, cudaStreamNonBlocking) != cudaSuccess) return nullptr;
+    if (cudaStreamCreateWithPriority(&st, cudaStreamNonBlocking, greatest) != cudaSuccess)
+      return nullptr;
     for (auto& e : ss.ev)
       if (cudaEventCreateWithFlags(&e, cudaEventDisableTiming) != cudaSuccess) return nullptr;
     ss.stream = st;

@@ -24,13 +24,12 @@ namespace {
 constexpr int SCAN_THREADS = 128;
 constexpr int SCAN_WARPS = SCAN_THREADS / 32;
 constexpr int MCH = 2;          // 4-element state chunks per thread: S <= 4 * 128 * MCH = 1024
-constexpr int KMAX = 32;
 
 struct Smem {
-  float* s;        // [S]     state
+  float* s;        // [S]     state (read back by nothing in the step loop; kept for debugging layout)
   float* F;        // [10][S] Fz then Fh, feature-major
-  float* d;        // [2][KMAX] residual dots (double-buffered)
-  float* gpart;    // [2][SCAN_WARPS] gate partial sums
+  float* gpart;    // [2][SCAN_WARPS] gate partial sums (double-buffered)
+  float* red;      // [2][SCAN_WARPS][32] residual-dot partial sums after the warp reduce-scatter
   int* cid;        // [L][K]
   float* clp;      // [L][K]
   float* top;      // [L][3]  l_i(c_0), l_i(c_1), l_i(c_3)
@@ -41,15 +40,16 @@ struct Smem {
   float* bsum;     // [nblk]  residual block sums
   float* misc;     // [16]
   int* imisc;      // [16]
-  float* U;        // [ubuf][K][S] residual rows of the candidates (one or two positions)
-  float* Tc;       // [2][K][2S] token-share rows of a position's candidates (when they fit)
+  float* U;        // [nbuf][K][S]  residual rows of a position's candidates
+  float* Tc;       // [nbuf][K][2S] token-share rows of the previous position's candidates
+  uint64_t* full;  // [nbuf] mbarriers: the bulk copies of a buffer have landed
 };
 
 __host__ __device__ inline size_t align16(size_t x) { return (x + 15) & ~size_t(15); }
 
 constexpr int RES_BLOCK = 256;  // residual-sampling block: 32 lanes x 8 ids
 
-__host__ __device__ inline size_t smem_layout(int L, int K, int S, int V, int ubuf, int tcand,
+__host__ __device__ inline size_t smem_layout(int L, int K, int S, int V, int nbuf, int tcand,
                                               char* base, Smem* sm) {
   size_t off = 0;
   auto take = [&](size_t bytes) {
@@ -60,8 +60,8 @@ __host__ __device__ inline size_t smem_layout(int L, int K, int S, int V, int ub
   const int nblk = (V + RES_BLOCK - 1) / RES_BLOCK;
   char* p_s = take(sizeof(float) * S);
   char* p_F = take(sizeof(float) * 10 * S);
-  char* p_d = take(sizeof(float) * 2 * KMAX);
   char* p_g = take(sizeof(float) * 2 * SCAN_WARPS);
+  char* p_red = take(sizeof(float) * 2 * SCAN_WARPS * 32);
   char* p_cid = take(sizeof(int) * L * K);
   char* p_clp = take(sizeof(float) * L * K);
   char* p_top = take(sizeof(float) * L * 3);
@@ -72,56 +72,85 @@ __host__ __device__ inline size_t smem_layout(int L, int K, int S, int V, int ub
   char* p_bsum = take(sizeof(float) * nblk);
   char* p_misc = take(sizeof(float) * 16);
   char* p_imisc = take(sizeof(int) * 16);
-  char* p_U = take(sizeof(float) * ubuf * K * S);
-  char* p_Tc = take(tcand ? sizeof(float) * 2 * K * 2 * S : 0);
+  char* p_U = take(sizeof(float) * nbuf * K * S);
+  char* p_Tc = take(tcand ? sizeof(float) * nbuf * K * 2 * S : 0);
+  char* p_full = take(sizeof(uint64_t) * 4);
   if (sm) {
-    sm->U = (float*)p_U;
-    sm->Tc = (float*)p_Tc;
-    sm->s = (float*)p_s; sm->F = (float*)p_F; sm->d = (float*)p_d; sm->gpart = (float*)p_g;
+    sm->full = (uint64_t*)p_full;
+    sm->s = (float*)p_s; sm->F = (float*)p_F; sm->gpart = (float*)p_g; sm->red = (float*)p_red;
     sm->cid = (int*)p_cid; sm->clp = (float*)p_clp; sm->top = (float*)p_top;
     sm->lprev = (float*)p_lprev; sm->sel = (int*)p_sel; sm->rank = (int*)p_rank;
     sm->ref = (float*)p_ref; sm->bsum = (float*)p_bsum; sm->misc = (float*)p_misc;
-    sm->imisc = (int*)p_imisc;
+    sm->imisc = (int*)p_imisc; sm->U = (float*)p_U; sm->Tc = (float*)p_Tc;
   }
   return off;
 }
 
-__device__ __forceinline__ void cp_async16(void* smem, const void* gmem) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(
-                   static_cast<uint32_t>(__cvta_generic_to_shared(smem))),
-               "l"(gmem)
-               : "memory");
-}
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
-// Wait until at most n of this thread's most recent cp.async groups are still pending.
-__device__ __forceinline__ void cp_async_wait_pending(int n) {
-  if (n <= 0) asm volatile("cp.async.wait_group 0;" ::: "memory");
-  else if (n == 1) asm volatile("cp.async.wait_group 1;" ::: "memory");
-  else if (n == 2) asm volatile("cp.async.wait_group 2;" ::: "memory");
-  else asm volatile("cp.async.wait_group 3;" ::: "memory");
-}
 __device__ __forceinline__ float4 ld4(const float* p) { return *reinterpret_cast<const float4*>(p); }
 __device__ __forceinline__ void prefetch_l2(const void* p) {
   asm volatile("prefetch.global.L2 [%0];" ::"l"(p));
 }
-
-// Residual rows U[c_k] of the K candidates into shared memory. Warp w owns candidates
-// k = w, w + 4, ...; lane l owns the 16-byte chunks l, l + 32, ... of each of its rows, and is
-// the only thread that later reads them, so its own cp.async wait suffices.
-__device__ __forceinline__ void fetch_U(float* Ush, const float* U, const int* ci, int K, int S) {
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  for (int k = warp; k < K; k += 4) {
-    const float* src = U + (size_t)ci[k] * S;
-    float* dst = Ush + (size_t)k * S;
-    for (int q = lane; q < S / 4; q += 32) cp_async16(dst + 4 * q, src + 4 * q);
+__device__ __forceinline__ uint32_t su32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(su32(bar)), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(su32(bar)), "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(su32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+constexpr long long SCAN_WAIT_LIMIT_CYCLES = 4000000000ll;   // about 2 s of SM clock
+// Bounded wait for a phase of an mbarrier; false when it expired.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const long long t0 = clock64();
+  for (unsigned n = 1;; ++n) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if ((n & 63) == 0 && clock64() - t0 > SCAN_WAIT_LIMIT_CYCLES) return false;
   }
 }
-// L2 prefetch of K vocabulary-table rows of `row_floats` floats.
-__device__ __forceinline__ void prefetch_rows(const float* table, const int* ci, int K, int row_floats) {
-  const int lines = (row_floats * 4 + 127) / 128;
-  for (int e = threadIdx.x; e < K * lines; e += SCAN_THREADS)
-    prefetch_l2(table + (size_t)ci[e / lines] * row_floats + (e % lines) * 32);
+// Bulk (TMA) copy of `bytes` (a multiple of 16, 16-byte aligned ends) completing on `bar`.
+__device__ __forceinline__ void bulk_copy(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+          su32(dst)),
+      "l"(src), "r"(bytes), "r"(su32(bar))
+      : "memory");
+}
+
+// Logistic function with the hardware exponential (relative error ~1e-6).
+__device__ __forceinline__ float sigmoid_fast(float x) { return __fdividef(1.f, 1.f + __expf(-x)); }
+
+// Warp reduce-scatter of NP values per lane: afterwards lane l holds the warp-wide sum of value
+// ((l >> 1) & 15) for NP = 16 and of value l for NP = 32.
+template <int NP>
+__device__ __forceinline__ float reduce_scatter(float (&v)[NP]) {
+  const int lane = threadIdx.x & 31;
+#pragma unroll
+  for (int m = 16, n = NP; n > 1; m >>= 1, n >>= 1) {
+    const bool upper = (lane & m) != 0;
+#pragma unroll
+    for (int j = 0; j < n / 2; ++j) {
+      const float send = upper ? v[j] : v[j + n / 2];
+      const float keep = upper ? v[j + n / 2] : v[j];
+      v[j] = keep + __shfl_xor_sync(FULL_MASK, send, m);
+    }
+  }
+  float r = v[0];
+  if (NP == 16) r += __shfl_xor_sync(FULL_MASK, r, 1);
+  return r;
 }
 
 __device__ __forceinline__ float load_logit(const void* base, int dt, size_t idx) {
@@ -129,33 +158,40 @@ __device__ __forceinline__ float load_logit(const void* base, int dt, size_t idx
   return reinterpret_cast<const float*>(base)[idx];
 }
 
-// Select over the K refined scores of one position, refined_k = clp[k] + gamma * d[k] read from
-// shared memory (identical arithmetic in every thread).
-__device__ __forceinline__ int select_rank(const float* clp, const float* d, float gamma, int K,
-                                           int mode, float u) {
+// Residual dot d_k of one position: the four warps' partial sums, added in a fixed order.
+__device__ __forceinline__ float dot_k(const float* red, int k) {
+  return ((red[k] + red[32 + k]) + red[64 + k]) + red[96 + k];
+}
+
+// Select with lane k holding refined score k (lanes >= K hold -inf); the same in every lane.
+// Greedy: argmax, the lowest rank on ties. Sample: the first rank whose cumulative softmax mass
+// exceeds u * total (warp prefix sums), else the last rank with mass.
+__device__ __forceinline__ int select_warp(float ref, int K, int mode, float u) {
+  const int lane = threadIdx.x & 31;
   if (mode == BRISK_SELECT_GREEDY) {
-    int best = 0;
-    float bv = clp[0] + gamma * d[0];
-    for (int k = 1; k < K; ++k) {
-      const float v = clp[k] + gamma * d[k];
-      if (v > bv) { bv = v; best = k; }
+    float bv = ref;
+    int bk = lane < K ? lane : 0x7fffffff;
+#pragma unroll
+    for (int off = 16; off; off >>= 1) {
+      const float ov = __shfl_xor_sync(FULL_MASK, bv, off);
+      const int ok = __shfl_xor_sync(FULL_MASK, bk, off);
+      if (ov > bv || (ov == bv && ok < bk)) { bv = ov; bk = ok; }
     }
-    return best;
+    return bk;
   }
-  float mx = clp[0] + gamma * d[0];
-  for (int k = 1; k < K; ++k) mx = fmaxf(mx, clp[k] + gamma * d[k]);
-  float tot = 0.f;
-  for (int k = 0; k < K; ++k) tot += expf(clp[k] + gamma * d[k] - mx);
-  const float target = u * tot;
-  float cum = 0.f;
-  int last = 0;
-  for (int k = 0; k < K; ++k) {
-    const float w = expf(clp[k] + gamma * d[k] - mx);
-    cum += w;
-    if (w > 0.f) last = k;
-    if (cum > target) return k;
+  const float mx = warp_max(ref);
+  const float w = lane < K ? expf(ref - mx) : 0.f;
+  float cum = w;
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const float o = __shfl_up_sync(FULL_MASK, cum, off);
+    if (lane >= off) cum += o;
   }
-  return last;
+  const float tot = __shfl_sync(FULL_MASK, cum, 31);
+  const unsigned hit = __ballot_sync(FULL_MASK, lane < K && cum > u * tot);
+  if (hit) return __ffs(hit) - 1;
+  const unsigned pos = __ballot_sync(FULL_MASK, w > 0.f);
+  return pos ? 31 - __clz(pos) : 0;
 }
 
 // pi_i(rank r) of the proposal law induced by the Select rule.
@@ -373,13 +409,201 @@ __device__ void verify_sequence(const ScanArgs& a, const Smem& sm, int b) {
     a.out_tokens[(size_t)b * L + t] = t < j ? sm.sel[t] : (t == j ? corr : -1);
 }
 
+// The sequential corrector over the positions of sequence b (Algorithm 1(b) loop). Thread t owns
+// the 4-element state chunks c = t + 128 m: it updates them, stages its own chunks of the
+// candidates' residual and token-share rows with cp.async (nbuf - 1 positions ahead; no other
+// thread reads them, so its own wait suffices), and contributes its partial residual dots, which
+// one warp reduce-scatter and one block barrier per position turn into the K dots.
+template <int NP>
+__device__ void corrector_loop(const ScanArgs& a, const Smem& sm, int b, int x0) {
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int L = a.L, K = a.K, S = a.S;
+  const size_t bL = (size_t)b * L;
+  const int nch = S / 4;
+  const int nbuf = a.ubuf, tcand = a.tcand;
+
+  float4 s4[MCH], wg4[MCH], gz4[MCH], gh4[MCH], tz4[MCH], th4[MCH];
+#pragma unroll
+  for (int m = 0; m < MCH; ++m) {
+    const int c = tid + m * SCAN_THREADS;
+    s4[m] = wg4[m] = gz4[m] = gh4[m] = tz4[m] = th4[m] = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (c < nch) {
+      const float4 g0 = ld4(a.G0 + (size_t)b * S + 4 * c), t0 = ld4(a.T0 + (size_t)x0 * S + 4 * c);
+      s4[m] = make_float4(tanhf(g0.x + t0.x), tanhf(g0.y + t0.y), tanhf(g0.z + t0.z),
+                          tanhf(g0.w + t0.w));                     // s_{-1} = u_0 = Init(h_c, E(x0))
+      wg4[m] = ld4(a.wg + 4 * c);
+      gz4[m] = ld4(a.G + bL * 2 * S + 4 * c);
+      gh4[m] = ld4(a.G + bL * 2 * S + S + 4 * c);
+      tz4[m] = ld4(a.Tzh + (size_t)x0 * 2 * S + 4 * c);           // token share of x_{-1} = x0
+      th4[m] = ld4(a.Tzh + (size_t)x0 * 2 * S + S + 4 * c);
+    }
+  }
+  float wgf[5];
+#pragma unroll
+  for (int f = 0; f < 5; ++f) wgf[f] = a.wg[S + f];
+  const float sig_alpha = sigmoidf_(a.alpha);
+
+  // The rows position j needs (the residual rows of its candidates and, when staged, the
+  // token-share rows of the previous position's candidates) arrive in buffer j % nbuf by bulk
+  // copies that thread 0 issues; everybody waits on that buffer's mbarrier.
+  const uint32_t u_bytes = (uint32_t)S * 4, t_bytes = (uint32_t)S * 8;
+  auto issue = [&](int j) {
+    if (tid != 0 || j >= L) return;
+    const int slot = j % nbuf;
+    float* Ub = sm.U + (size_t)slot * K * S;
+    float* Tb = sm.Tc + (size_t)slot * K * 2 * S;
+    const bool with_t = tcand && j > 0;
+    mbar_expect_tx(&sm.full[slot], K * (u_bytes + (with_t ? t_bytes : 0)));
+    for (int k = 0; k < K; ++k) {
+      bulk_copy(Ub + (size_t)k * S, a.U + (size_t)sm.cid[j * K + k] * S, u_bytes, &sm.full[slot]);
+      if (with_t)
+        bulk_copy(Tb + (size_t)k * 2 * S, a.Tzh + (size_t)sm.cid[(j - 1) * K + k] * 2 * S, t_bytes,
+                  &sm.full[slot]);
+    }
+  };
+  if (tid == 0) {
+    for (int q = 0; q < nbuf; ++q) mbar_init(&sm.full[q], 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  __syncthreads();
+  const int ahead = nbuf > 1 ? nbuf - 1 : 0;
+  for (int j = 0; j < (nbuf > 1 ? ahead : 1); ++j) issue(j);
+  // this thread's share of the L2 prefetch of a table row: fixed across positions
+  const int u_lines = (S * 4 + 127) / 128, t_lines = (S * 8 + 127) / 128;
+  const int pu_k = tid / u_lines, pu_l = tid % u_lines;
+  bool timed_out = false;
+
+  int prev = x0, prank = 0;
+  float u_cur = (a.select_mode == BRISK_SELECT_SAMPLE) ? a.u_sel[bL] : 0.f;
+  for (int i = 0; i < L; ++i) {
+    const int buf = i & 1;
+    const int* ci = sm.cid + i * K;
+    if (nbuf > 1) issue(i + ahead);
+    // L2 prefetch further ahead (and of the gathered token-share rows when they are not staged)
+    if (i + nbuf < L && pu_k < K) prefetch_l2(a.U + (size_t)ci[nbuf * K + pu_k] * S + pu_l * 32);
+    if (!tcand && i + 1 < L)
+      for (int e = tid; e < K * t_lines; e += SCAN_THREADS)
+        prefetch_l2(a.Tzh + (size_t)ci[e / t_lines] * 2 * S + (e % t_lines) * 32);
+    // confidence features of position i (App. C.2)
+    const float l0 = sm.top[i * 3 + 0];
+    float phi[5];
+    phi[0] = l0 - sm.top[i * 3 + 1];
+    phi[1] = l0 - sm.top[i * 3 + 2];
+    phi[2] = (prev == ci[0]) ? 1.f : 0.f;
+    phi[3] = (prev == ci[0] || prev == ci[1] || prev == ci[2] || prev == ci[3]) ? 1.f : 0.f;
+    phi[4] = l0 - sm.lprev[i * K + (i == 0 ? 0 : prank)];
+    // the rows of position i have landed
+    if (!mbar_wait(&sm.full[i % nbuf], (i / nbuf) & 1)) timed_out = true;
+    const float* Ub = sm.U + (size_t)(i % nbuf) * K * S;
+    // token share of the previous token (x0's came with the prologue)
+    if (i > 0) {
+      const float* Tp = tcand ? sm.Tc + ((size_t)(i % nbuf) * K + prank) * 2 * S
+                              : a.Tzh + (size_t)prev * 2 * S;
+#pragma unroll
+      for (int m = 0; m < MCH; ++m) {
+        const int c = tid + m * SCAN_THREADS;
+        if (c < nch) {
+          tz4[m] = ld4(Tp + 4 * c);
+          th4[m] = ld4(Tp + S + 4 * c);
+        }
+      }
+    }
+    // minimal-GRU step on this thread's chunks, its gate partial and its residual-dot partials
+    float gacc = 0.f;
+    float part[NP];
+#pragma unroll
+    for (int k = 0; k < NP; ++k) part[k] = 0.f;
+#pragma unroll
+    for (int m = 0; m < MCH; ++m) {
+      const int c = tid + m * SCAN_THREADS;
+      if (c < nch) {
+        float zp[4] = {gz4[m].x + tz4[m].x, gz4[m].y + tz4[m].y, gz4[m].z + tz4[m].z,
+                       gz4[m].w + tz4[m].w};
+        float hp[4] = {gh4[m].x + th4[m].x, gh4[m].y + th4[m].y, gh4[m].z + th4[m].z,
+                       gh4[m].w + th4[m].w};
+#pragma unroll
+        for (int f = 0; f < 5; ++f) {
+          const float4 fz = ld4(sm.F + (size_t)f * S + 4 * c);
+          const float4 fh = ld4(sm.F + (size_t)(5 + f) * S + 4 * c);
+          zp[0] = fmaf(fz.x, phi[f], zp[0]); zp[1] = fmaf(fz.y, phi[f], zp[1]);
+          zp[2] = fmaf(fz.z, phi[f], zp[2]); zp[3] = fmaf(fz.w, phi[f], zp[3]);
+          hp[0] = fmaf(fh.x, phi[f], hp[0]); hp[1] = fmaf(fh.y, phi[f], hp[1]);
+          hp[2] = fmaf(fh.z, phi[f], hp[2]); hp[3] = fmaf(fh.w, phi[f], hp[3]);
+        }
+        float sv[4] = {s4[m].x, s4[m].y, s4[m].z, s4[m].w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const float z = sigmoid_fast(zp[e]);
+          sv[e] = (1.f - z) * sv[e] + z * hp[e];
+        }
+        s4[m] = make_float4(sv[0], sv[1], sv[2], sv[3]);
+        gacc = fmaf(wg4[m].x, sv[0], gacc);
+        gacc = fmaf(wg4[m].y, sv[1], gacc);
+        gacc = fmaf(wg4[m].z, sv[2], gacc);
+        gacc = fmaf(wg4[m].w, sv[3], gacc);
+#pragma unroll
+        for (int k = 0; k < NP; ++k) {
+          if (k < K) {
+            const float4 u = ld4(Ub + (size_t)k * S + 4 * c);
+            part[k] = fmaf(u.x, sv[0], fmaf(u.y, sv[1], fmaf(u.z, sv[2], fmaf(u.w, sv[3], part[k]))));
+          }
+        }
+      }
+    }
+    // hidden and position shares of the next position: plain loads first used in the next step
+    if (i + 1 < L) {
+      const float* Gn = a.G + (bL + i + 1) * 2 * S;
+#pragma unroll
+      for (int m = 0; m < MCH; ++m) {
+        const int c = tid + m * SCAN_THREADS;
+        if (c < nch) {
+          gz4[m] = ld4(Gn + 4 * c);
+          gh4[m] = ld4(Gn + S + 4 * c);
+        }
+      }
+    }
+    // block reduction: residual dots by one reduce-scatter per warp, gate partial by a warp sum
+    const float r = reduce_scatter<NP>(part);
+    const int v = NP == 16 ? ((lane >> 1) & 15) : lane;
+    float* red = sm.red + buf * SCAN_WARPS * 32;
+    if (v < K && (NP == 32 || (lane & 1) == 0)) red[warp * 32 + v] = r;
+    gacc = warp_sum(gacc);
+    if (lane == 0) sm.gpart[buf * SCAN_WARPS + warp] = gacc;
+    __syncthreads();
+    if (nbuf == 1) issue(i + 1);   // every thread is done with the single buffer
+    // gate, refined scores (lane k: candidate k) and Select, identically in every warp
+    float gate = a.b_g;
+    for (int w = 0; w < SCAN_WARPS; ++w) gate += sm.gpart[buf * SCAN_WARPS + w];
+#pragma unroll
+    for (int f = 0; f < 5; ++f) gate = fmaf(wgf[f], phi[f], gate);
+    const float gamma = sig_alpha * sigmoid_fast(gate);
+    const float* clp = sm.clp + i * K;
+    const float ref = lane < K ? clp[lane] + gamma * dot_k(red, lane) : -INFINITY;
+    const int pick = select_warp(ref, K, a.select_mode, u_cur);
+    if (warp == 0 && lane < K) {
+      sm.ref[i * K + lane] = ref;
+      a.refined[(bL + i) * K + lane] = ref;
+    }
+    if (a.select_mode == BRISK_SELECT_SAMPLE && i + 1 < L) u_cur = a.u_sel[bL + i + 1];
+    prank = pick;
+    prev = ci[pick];
+    if (tid == 0) {
+      sm.sel[i] = prev;
+      sm.rank[i] = pick;
+      a.sel_tokens[bL + i] = prev;
+    }
+  }
+  if (timed_out && lane == 0) set_status(a.status, BRISK_ERR_TIMEOUT);
+  // every copy that was issued has been waited for above (the last one at position L - 1)
+}
+
 __global__ void __launch_bounds__(SCAN_THREADS)
 scan_kernel(const __grid_constant__ ScanArgs a) {
   extern __shared__ __align__(16) char smem_raw[];
   Smem sm;
   smem_layout(a.L, a.K, a.S, a.V, a.ubuf, a.tcand, smem_raw, &sm);
   const int b = blockIdx.x;
-  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int tid = threadIdx.x;
   const int L = a.L, K = a.K, S = a.S, V = a.V;
   const size_t bL = (size_t)b * L;
 
@@ -426,197 +650,8 @@ scan_kernel(const __grid_constant__ ScanArgs a) {
       sm.F[f * S + j] = a.Fz[e];
       sm.F[(5 + f) * S + j] = a.Fh[e];
     }
-    // this thread owns the 4-element state chunks c = tid + 128 m
-    const int nch = S / 4;
-    float4 s4[MCH], wg4[MCH], gz4[MCH], gh4[MCH], tz4[MCH], th4[MCH];
-#pragma unroll
-    for (int m = 0; m < MCH; ++m) {
-      const int c = tid + m * SCAN_THREADS;
-      s4[m] = wg4[m] = gz4[m] = gh4[m] = tz4[m] = th4[m] = make_float4(0.f, 0.f, 0.f, 0.f);
-      if (c < nch) {
-        const float4 g0 = ld4(a.G0 + (size_t)b * S + 4 * c), t0 = ld4(a.T0 + (size_t)x0 * S + 4 * c);
-        s4[m] = make_float4(tanhf(g0.x + t0.x), tanhf(g0.y + t0.y), tanhf(g0.z + t0.z),
-                            tanhf(g0.w + t0.w));
-        wg4[m] = ld4(a.wg + 4 * c);
-        gz4[m] = ld4(a.G + bL * 2 * S + 4 * c);
-        gh4[m] = ld4(a.G + bL * 2 * S + S + 4 * c);
-        tz4[m] = ld4(a.Tzh + (size_t)x0 * 2 * S + 4 * c);        // token share of x_{-1} = x0
-        th4[m] = ld4(a.Tzh + (size_t)x0 * 2 * S + S + 4 * c);
-      }
-    }
-    float wgf[5];
-#pragma unroll
-    for (int f = 0; f < 5; ++f) wgf[f] = a.wg[S + f];
-    const float sig_alpha = sigmoidf_(a.alpha);
-    // residual rows of positions 0 (and 1) into shared memory; one cp.async group per batch,
-    // committed even when empty, so that the group counts below are the same at every step
-    const int ubuf = a.ubuf, tcand = a.tcand;
-    fetch_U(sm.U, a.U, sm.cid, K, S);
-    cp_async_commit();
-    if (ubuf == 2) {
-      if (L > 1) fetch_U(sm.U + (size_t)K * S, a.U, sm.cid + K, K, S);
-      cp_async_commit();
-    }
-    __syncthreads();
-
-    int prev = x0, prank = 0;
-    float u_next = (a.select_mode == BRISK_SELECT_SAMPLE) ? a.u_sel[bL] : 0.f;
-    for (int i = 0; i < L; ++i) {
-      const int buf = i & 1;
-      const int* ci = sm.cid + i * K;
-      // the token-share rows of the next position's previous token are among this position's
-      // candidates: stage them all (own chunks only) in shared memory, or pull them into L2
-      if (tcand) {
-        if (i + 1 < L) {
-          float* Tb = sm.Tc + (size_t)buf * K * 2 * S;
-          for (int k = 0; k < K; ++k) {
-            const float* src = a.Tzh + (size_t)ci[k] * 2 * S;
-#pragma unroll
-            for (int m = 0; m < MCH; ++m) {
-              const int c = tid + m * SCAN_THREADS;
-              if (c < nch) {
-                cp_async16(Tb + (size_t)k * 2 * S + 4 * c, src + 4 * c);
-                cp_async16(Tb + (size_t)k * 2 * S + S + 4 * c, src + S + 4 * c);
-              }
-            }
-          }
-        }
-        cp_async_commit();
-      } else if (i + 1 < L) {
-        prefetch_rows(a.Tzh, ci, K, 2 * S);
-      }
-      if (i + ubuf < L) prefetch_rows(a.U, ci + ubuf * K, K, S);
-      float* Ucur = sm.U + (size_t)(ubuf == 2 ? (i & 1) : 0) * K * S;
-      // confidence features of position i (App. C.2)
-      const float l0 = sm.top[i * 3 + 0];
-      float phi[5];
-      phi[0] = l0 - sm.top[i * 3 + 1];
-      phi[1] = l0 - sm.top[i * 3 + 2];
-      phi[2] = (prev == ci[0]) ? 1.f : 0.f;
-      phi[3] = (prev == ci[0] || prev == ci[1] || prev == ci[2] || prev == ci[3]) ? 1.f : 0.f;
-      phi[4] = l0 - sm.lprev[i * K + (i == 0 ? 0 : prank)];
-      // token share of the previous token (x0's was loaded in the prologue)
-      if (i > 0) {
-        if (tcand) {
-          const float* Tp = sm.Tc + ((size_t)((i - 1) & 1) * K + prank) * 2 * S;
-#pragma unroll
-          for (int m = 0; m < MCH; ++m) {
-            const int c = tid + m * SCAN_THREADS;
-            if (c < nch) {
-              tz4[m] = ld4(Tp + 4 * c);
-              th4[m] = ld4(Tp + S + 4 * c);
-            }
-          }
-        } else {
-          const float* Ti = a.Tzh + (size_t)prev * 2 * S;
-#pragma unroll
-          for (int m = 0; m < MCH; ++m) {
-            const int c = tid + m * SCAN_THREADS;
-            if (c < nch) {
-              tz4[m] = ld4(Ti + 4 * c);
-              th4[m] = ld4(Ti + S + 4 * c);
-            }
-          }
-        }
-      }
-      // minimal-GRU step on this thread's state chunks
-      float gacc = 0.f;
-#pragma unroll
-      for (int m = 0; m < MCH; ++m) {
-        const int c = tid + m * SCAN_THREADS;
-        if (c < nch) {
-          float zp[4] = {gz4[m].x + tz4[m].x, gz4[m].y + tz4[m].y, gz4[m].z + tz4[m].z,
-                         gz4[m].w + tz4[m].w};
-          float hp[4] = {gh4[m].x + th4[m].x, gh4[m].y + th4[m].y, gh4[m].z + th4[m].z,
-                         gh4[m].w + th4[m].w};
-#pragma unroll
-          for (int f = 0; f < 5; ++f) {
-            const float4 fz = ld4(sm.F + (size_t)f * S + 4 * c);
-            const float4 fh = ld4(sm.F + (size_t)(5 + f) * S + 4 * c);
-            zp[0] = fmaf(fz.x, phi[f], zp[0]); zp[1] = fmaf(fz.y, phi[f], zp[1]);
-            zp[2] = fmaf(fz.z, phi[f], zp[2]); zp[3] = fmaf(fz.w, phi[f], zp[3]);
-            hp[0] = fmaf(fh.x, phi[f], hp[0]); hp[1] = fmaf(fh.y, phi[f], hp[1]);
-            hp[2] = fmaf(fh.z, phi[f], hp[2]); hp[3] = fmaf(fh.w, phi[f], hp[3]);
-          }
-          float sv[4] = {s4[m].x, s4[m].y, s4[m].z, s4[m].w};
-#pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            const float z = sigmoidf_(zp[e]);
-            sv[e] = (1.f - z) * sv[e] + z * hp[e];
-          }
-          s4[m] = make_float4(sv[0], sv[1], sv[2], sv[3]);
-          *reinterpret_cast<float4*>(sm.s + 4 * c) = s4[m];
-          gacc = fmaf(wg4[m].x, sv[0], gacc);
-          gacc = fmaf(wg4[m].y, sv[1], gacc);
-          gacc = fmaf(wg4[m].z, sv[2], gacc);
-          gacc = fmaf(wg4[m].w, sv[3], gacc);
-        }
-      }
-      // hidden and position shares of the next position: plain loads whose values are first
-      // used in the next step, so they stay in flight meanwhile
-      if (i + 1 < L) {
-        const float* Gn = a.G + (bL + i + 1) * 2 * S;
-#pragma unroll
-        for (int m = 0; m < MCH; ++m) {
-          const int c = tid + m * SCAN_THREADS;
-          if (c < nch) {
-            gz4[m] = ld4(Gn + 4 * c);
-            gh4[m] = ld4(Gn + S + 4 * c);
-          }
-        }
-      }
-      gacc = warp_sum(gacc);
-      if (lane == 0) sm.gpart[buf * SCAN_WARPS + warp] = gacc;
-      // this lane's residual rows of position i have landed (groups committed after them: the
-      // next position's rows, and this and the previous position's token-share batches)
-      if (tcand) cp_async_wait_pending(ubuf == 2 ? (i == 0 ? 2 : 3) : 1);
-      else cp_async_wait_pending(ubuf == 2 ? 1 : 0);
-      __syncthreads();
-      // residual dots d_k = <s, U[c_k]>, one warp per candidate, rows from shared memory
-      for (int k = warp; k < K; k += SCAN_WARPS) {
-        const float4* Uk = reinterpret_cast<const float4*>(Ucur + (size_t)k * S);
-        const float4* s4 = reinterpret_cast<const float4*>(sm.s);
-        float acc = 0.f;
-        for (int q = lane; q < S / 4; q += 32) {
-          const float4 u = Uk[q], v = s4[q];
-          acc = fmaf(u.x, v.x, acc);
-          acc = fmaf(u.y, v.y, acc);
-          acc = fmaf(u.z, v.z, acc);
-          acc = fmaf(u.w, v.w, acc);
-        }
-        acc = warp_sum(acc);
-        if (lane == 0) sm.d[buf * KMAX + k] = acc;
-      }
-      // residual rows of position i + ubuf into the buffer just read (each lane refills exactly
-      // the chunks it read itself)
-      if (i + ubuf < L) fetch_U(Ucur, a.U, ci + ubuf * K, K, S);
-      cp_async_commit();
-      __syncthreads();
-      // gate, refined scores and Select (every thread, identical arithmetic)
-      float gate = a.b_g;
-      for (int w = 0; w < SCAN_WARPS; ++w) gate += sm.gpart[buf * SCAN_WARPS + w];
-#pragma unroll
-      for (int f = 0; f < 5; ++f) gate = fmaf(wgf[f], phi[f], gate);
-      const float gamma = sig_alpha * sigmoidf_(gate);
-      const float* clp = sm.clp + i * K;
-      const float* dk = sm.d + buf * KMAX;
-      const int pick = select_rank(clp, dk, gamma, K, a.select_mode, u_next);
-      if (tid < K) {
-        const float ref = clp[tid] + gamma * dk[tid];
-        sm.ref[i * K + tid] = ref;
-        a.refined[(bL + i) * K + tid] = ref;
-      }
-      if (a.select_mode == BRISK_SELECT_SAMPLE && i + 1 < L) u_next = a.u_sel[bL + i + 1];
-      // this thread's token-share chunks of this position's candidates have landed
-      if (tcand) cp_async_wait_pending(1);
-      prank = pick;
-      prev = ci[pick];
-      if (tid == 0) {
-        sm.sel[i] = prev;
-        sm.rank[i] = pick;
-        a.sel_tokens[bL + i] = prev;
-      }
-    }
+    if (K + 1 <= 16) corrector_loop<16>(a, sm, b, x0);
+    else corrector_loop<32>(a, sm, b, x0);
     __syncthreads();
   } else {
     // verify alone: recover each selection's rank in its candidate list
@@ -636,18 +671,18 @@ scan_kernel(const __grid_constant__ ScanArgs a) {
 
 constexpr size_t SCAN_SMEM_LIMIT = 227 * 1024;
 
-// Shared-memory plan: double-buffered residual rows and staged token-share rows when they fit,
-// else fewer buffers.
-void scan_plan(int L, int K, int S, int V, int* ubuf, int* tcand) {
-  const int plans[3][2] = {{2, 1}, {2, 0}, {1, 0}};
+// Shared-memory plan: stage the token-share rows and prefetch two positions ahead when that
+// fits, else less.
+void scan_plan(int L, int K, int S, int V, int* nbuf, int* tcand) {
+  const int plans[5][2] = {{3, 1}, {2, 1}, {3, 0}, {2, 0}, {1, 0}};
   for (const auto& p : plans) {
     if (smem_layout(L, K, S, V, p[0], p[1], nullptr, nullptr) <= SCAN_SMEM_LIMIT) {
-      *ubuf = p[0];
+      *nbuf = p[0];
       *tcand = p[1];
       return;
     }
   }
-  *ubuf = 1;
+  *nbuf = 1;
   *tcand = 0;
 }
 
