@@ -315,8 +315,10 @@ def run_ours(args):
     g1 = torch.cuda.Event(enable_timing=True)
     wall0 = time.time()
     g0.record(stream)
+    h0 = time.perf_counter()
     for s in range(args.warmup, nsteps):
         step(s)
+    host_enqueue_s = time.perf_counter() - h0
     g1.record(stream)
     torch.cuda.synchronize()
     wall1 = time.time()
@@ -396,6 +398,7 @@ def run_ours(args):
         "gpu_launches": brisk.kernels_per_tail(tail.dims) * args.steps,
         "clocks": sampler.summary(wall0, wall1),
         "committed_tokens_per_s": committed_all / elapsed_max,
+        "host_enqueue_us_per_step": 1e6 * host_enqueue_s / args.steps,
         "accepted_per_sequence_block": tokens / (wl.B * world * args.steps),
     }
     print(json.dumps(line))

@@ -118,9 +118,9 @@ typedef struct brisk_tail_io {
   int32_t *next_anchor;     /* optional [B] last committed token (anchor of the next block) */
 } brisk_tail_io;
 
-/* Optional timing hooks: cudaEvent_t handles (as void*) recorded on `stream` right before and
- * right after the two vocabulary-sweep kernels of brisk_decode_tail (proposal rows, verifier
- * rows). NULL fields are skipped. */
+/* Optional timing hooks: cudaEvent_t handles (as void*) recorded right before and right after
+ * the two vocabulary-sweep kernels of brisk_decode_tail (proposal rows on `stream`, verifier
+ * rows on the library's side stream). NULL fields are skipped. */
 typedef struct brisk_events {
   void *sweep_q_begin, *sweep_q_end, *sweep_p_begin, *sweep_p_end;
 } brisk_events;
@@ -198,11 +198,12 @@ brisk_status brisk_verify_block(const brisk_dims *dims, const void *logits_p,
 
 /* Steps 1-3 for one block step (Algorithm 1(b) lines after the backbone pass): the same results,
  * bit for bit, as brisk_topk_candidates + brisk_corrector_select + brisk_verify_block on the same
- * inputs. The corrector needs only the proposal candidates, so it runs on a library side stream
- * while the verifier rows are swept; the call still only enqueues work and the results are
- * ordered on `stream` (the side stream forks from and joins back to it, also under graph
- * capture). The first call on a device creates the side stream and its events: make it before
- * any stream capture. Calls from several host threads are serialised while they enqueue.
+ * inputs. The corrector needs only the proposal candidates, so the verifier rows are swept on a
+ * library side stream while the corrector runs (and the hidden-state products run on another
+ * side stream during the proposal sweep); the call still only enqueues work and the results are
+ * ordered on `stream` (the side streams fork from and join back to it, also under graph
+ * capture). The first call on a device creates the side streams and their events: make it
+ * before any stream capture. Calls from several host threads are serialised while they enqueue.
  * `ev` may be NULL. */
 brisk_status brisk_decode_tail(const brisk_dims *dims, const brisk_params *params,
                                const void *tables, const brisk_tail_io *io, int32_t select_mode,

@@ -30,16 +30,17 @@ inline size_t esize(int dt) { return dt == BRISK_DT_BF16 ? 2 : 4; }
 struct WsLayout {
   size_t status, counters, part_val, part_id, part_m, part_s, argmax_p, lse_p;
   size_t cand_ids, cand_logprob, lse_q, sel, refined, Hm, G, G0, total;
-  int nchunk, KP;
+  int nchunk_q, nchunk_p, KP;   // chunks per proposal row (row layout) and verifier row (split)
 };
 
 WsLayout ws_layout(const brisk_dims* d) {
   WsLayout w{};
   const size_t BL = (size_t)d->B * d->L;
   const size_t S = 2 * (size_t)d->r;
-  w.nchunk = sweep_chunks((int)BL, d->V, d->logits_dtype, 0);
+  w.nchunk_q = sweep_chunks((int)BL, d->V, d->logits_dtype, SWEEP_ROWS);
+  w.nchunk_p = sweep_chunks((int)BL, d->V, d->logits_dtype, SWEEP_SPLIT);
   w.KP = kp_for(d->K);
-  const size_t np = 2 * BL * w.nchunk;
+  const size_t np = BL * (size_t)(w.nchunk_q + w.nchunk_p);
   size_t o = 0;
   auto take = [&](size_t bytes) { const size_t r = o; o = up(o + bytes); return r; };
   w.status = take(ALIGN);
@@ -127,8 +128,7 @@ brisk_status clear_ws(const WsLayout& w, const brisk_dims* d, void* ws, cudaStre
 SweepSeg make_seg(const WsLayout& w, void* ws, int seg, const void* logits, int rows, int kout,
                   int32_t* out_ids, float* out_logprob, float* out_lse) {
   SweepSeg s{};
-  const size_t np = (size_t)rows * w.nchunk;
-  const size_t off = seg * np;
+  const size_t off = seg ? (size_t)rows * w.nchunk_q : 0;   // segment 1 follows segment 0
   s.logits = logits;
   s.rows = rows;
   s.kout = kout;
@@ -183,8 +183,9 @@ brisk_status hidden_products(const brisk_dims* d, const brisk_params* p, const v
 // A side stream per device (created on the first fused call on that device) and the events that
 // fork work onto it and join it back, so that one call can run independent stages concurrently.
 struct SideStream {
-  cudaStream_t stream = nullptr;
-  cudaEvent_t ev[3] = {nullptr, nullptr, nullptr};
+  cudaStream_t hi = nullptr;   // highest priority: the hidden-state products
+  cudaStream_t lo = nullptr;   // lowest priority: the verifier-row sweep
+  cudaEvent_t ev[4] = {nullptr, nullptr, nullptr, nullptr};
 };
 constexpr int MAX_DEVICES = 256;
 std::mutex g_side_mu;
@@ -194,17 +195,17 @@ SideStream* side_stream() {
   int dev = -1;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= MAX_DEVICES) return nullptr;
   SideStream& ss = g_side[dev];
-  if (!ss.stream) {
-    // highest priority: when a stage on the side stream becomes ready together with a sweep on
-    // the caller's stream, its blocks are placed first and the sweep fills the remaining room
+  if (!ss.hi) {
     int least = 0, greatest = 0;
     if (cudaDeviceGetStreamPriorityRange(&least, &greatest) != cudaSuccess) return nullptr;
-    cudaStream_t st = nullptr;
-    if (cudaStreamCreateWithPriority(&st, cudaStreamNonBlocking, greatest) != cudaSuccess)
+    cudaStream_t hi = nullptr, lo = nullptr;
+    if (cudaStreamCreateWithPriority(&hi, cudaStreamNonBlocking, greatest) != cudaSuccess ||
+        cudaStreamCreateWithPriority(&lo, cudaStreamNonBlocking, least) != cudaSuccess)
       return nullptr;
     for (auto& e : ss.ev)
       if (cudaEventCreateWithFlags(&e, cudaEventDisableTiming) != cudaSuccess) return nullptr;
-    ss.stream = st;
+    ss.lo = lo;
+    ss.hi = hi;
   }
   return &ss;
 }
@@ -325,7 +326,8 @@ brisk_status brisk_topk_candidates(const brisk_dims* d, const void* logits_q, in
   a.seg[0] = make_seg(w, ws, 0, logits_q, d->B * d->L, d->K, cand_ids, cand_logprob, lse_q);
   a.nseg = 1;
   a.V = d->V;
-  a.nchunk = w.nchunk;
+  a.mode = SWEEP_ROWS;
+  a.nchunk = w.nchunk_q;
   a.KP = w.KP;
   a.dtype = d->logits_dtype;
   a.status = at<int32_t>(ws, w.status);
@@ -390,7 +392,8 @@ brisk_status brisk_verify_block(const brisk_dims* d, const void* logits_p, const
                        at<float>(ws, w.lse_p));
   sw.nseg = 1;
   sw.V = d->V;
-  sw.nchunk = w.nchunk;
+  sw.mode = SWEEP_SPLIT;
+  sw.nchunk = w.nchunk_p;
   sw.KP = w.KP;
   sw.dtype = d->logits_dtype;
   sw.status = at<int32_t>(ws, w.status);
@@ -440,37 +443,51 @@ brisk_status brisk_decode_tail(const brisk_dims* d, const brisk_params* p, const
   int32_t* sel = io->sel_tokens ? io->sel_tokens : at<int32_t>(ws, w.sel);
   float* refined = io->refined ? io->refined : at<float>(ws, w.refined);
 
-  // Schedule (A = caller's stream, B = side stream):
-  //   A: proposal-row sweep ............ verifier-row sweep ... join ... verification
-  //   B: hidden-state products ... join ... corrector scan
+  // Schedule. A = the caller's stream, H / W = side streams of highest / lowest priority:
+  //   H: hidden-state products --------.
+  //   A: proposal-row sweep ----------- join -> corrector scan ---- join -> verification
+  //   W:                      `-> verifier-row sweep ----------------'
   // The corrector needs only the proposal candidates and the hidden products; the verifier rows
-  // are needed only by the verification, so the corrector runs under the second sweep.
+  // are needed only by the verification, so the corrector runs while the verifier rows are
+  // swept. Priorities decide which ready blocks the GPU places first: the products before the
+  // proposal sweep, the corrector before the verifier sweep (which fills the remaining room).
   std::lock_guard<std::mutex> lock(g_side_mu);
   SideStream* ss = side_stream();
   if (!ss) return BRISK_ERR_CUDA;
-  cudaStream_t sb = ss->stream;
   BRISK_CUDA(cudaEventRecord(ss->ev[0], st));
-  BRISK_CUDA(cudaStreamWaitEvent(sb, ss->ev[0], 0));
-  s = hidden_products(d, p, tables, io->hidden, io->h_ctx, w, ws, sb, 2);
+  BRISK_CUDA(cudaStreamWaitEvent(ss->hi, ss->ev[0], 0));
+  s = hidden_products(d, p, tables, io->hidden, io->h_ctx, w, ws, ss->hi, 2);
   if (s != BRISK_OK) return s;
+  BRISK_CUDA(cudaEventRecord(ss->ev[1], ss->hi));
 
   SweepLaunch sq{};
   sq.seg[0] = make_seg(w, ws, 0, io->logits_q, BL, d->K, cand_ids, cand_lp, lse_q);
   sq.nseg = 1;
   sq.V = d->V;
-  sq.nchunk = w.nchunk;
+  sq.mode = SWEEP_ROWS;
+  sq.nchunk = w.nchunk_q;
   sq.KP = w.KP;
   sq.dtype = d->logits_dtype;
   sq.status = at<int32_t>(ws, w.status);
   SweepLaunch sp = sq;
   sp.seg[0] = make_seg(w, ws, 1, io->logits_p, BL, 1, at<int32_t>(ws, w.argmax_p), nullptr,
                        at<float>(ws, w.lse_p));
+  sp.mode = SWEEP_SPLIT;
+  sp.nchunk = w.nchunk_p;
   if (ev && ev->sweep_q_begin) BRISK_CUDA(cudaEventRecord(static_cast<cudaEvent_t>(ev->sweep_q_begin), st));
   BRISK_CUDA(launch_sweep(sq, st));
   if (ev && ev->sweep_q_end) BRISK_CUDA(cudaEventRecord(static_cast<cudaEvent_t>(ev->sweep_q_end), st));
-  BRISK_CUDA(cudaEventRecord(ss->ev[1], st));
+  BRISK_CUDA(cudaEventRecord(ss->ev[2], st));
 
-  BRISK_CUDA(cudaStreamWaitEvent(sb, ss->ev[1], 0));
+  // verifier rows on the low-priority stream, after the proposal sweep
+  BRISK_CUDA(cudaStreamWaitEvent(ss->lo, ss->ev[2], 0));
+  if (ev && ev->sweep_p_begin) BRISK_CUDA(cudaEventRecord(static_cast<cudaEvent_t>(ev->sweep_p_begin), ss->lo));
+  BRISK_CUDA(launch_sweep(sp, ss->lo));
+  if (ev && ev->sweep_p_end) BRISK_CUDA(cudaEventRecord(static_cast<cudaEvent_t>(ev->sweep_p_end), ss->lo));
+  BRISK_CUDA(cudaEventRecord(ss->ev[3], ss->lo));
+
+  // the corrector on the caller's stream, once the hidden products are done
+  BRISK_CUDA(cudaStreamWaitEvent(st, ss->ev[1], 0));
   ScanArgs a = scan_args(d, p, tables, w, ws);
   a.select_mode = select_mode;
   a.verify_mode = verify_mode;
@@ -483,13 +500,8 @@ brisk_status brisk_decode_tail(const brisk_dims* d, const brisk_params* p, const
   a.u_sel = io->u_sel;
   a.sel_tokens = sel;
   a.refined = refined;
-  BRISK_CUDA(launch_scan(a, sb));
-  BRISK_CUDA(cudaEventRecord(ss->ev[2], sb));
-
-  if (ev && ev->sweep_p_begin) BRISK_CUDA(cudaEventRecord(static_cast<cudaEvent_t>(ev->sweep_p_begin), st));
-  BRISK_CUDA(launch_sweep(sp, st));
-  if (ev && ev->sweep_p_end) BRISK_CUDA(cudaEventRecord(static_cast<cudaEvent_t>(ev->sweep_p_end), st));
-  BRISK_CUDA(cudaStreamWaitEvent(st, ss->ev[2], 0));
+  BRISK_CUDA(launch_scan(a, st));
+  BRISK_CUDA(cudaStreamWaitEvent(st, ss->ev[3], 0));
 
   ScanArgs v = scan_args(d, nullptr, nullptr, w, ws);
   v.select_mode = select_mode;

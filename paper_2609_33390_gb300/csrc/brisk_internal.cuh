@@ -5,6 +5,7 @@
 #include <cuda_bf16.h>
 #include <stdint.h>
 #include <math.h>
+#include <atomic>
 
 #include "../../include/brisk.h"
 
@@ -141,6 +142,32 @@ __device__ __forceinline__ void warp_lse_combine(float& m, float& s) {
   s = t;
 }
 
+// Shared-memory carveouts (KB) the kernels ask for. An SM cannot change its L1/shared split
+// while a CTA is resident, and the first kernel to land on an idle SM sets it, so a kernel that
+// runs beside another one (the sweep beside the dense products, the verifier-row sweep beside
+// the corrector) must leave room in its split for the other's CTAs. Everything not carved out
+// is L1, which holds the sweep's loads in flight: the sweep is fastest with a small split.
+constexpr int CARVEOUT_SMALL_KB = 64;    // sweep (2 KB a CTA), corrector, verification
+constexpr int CARVEOUT_GEMM_KB = 132;    // a dense-product CTA (up to 97 KB) beside six sweep CTAs
+
+template <typename Kernel>
+inline cudaError_t prefer_carveout(Kernel kernel, int kb) {
+  static std::atomic<unsigned long long> done{0};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  const unsigned long long bit = 1ull << (dev & 63);
+  if (done.load(std::memory_order_relaxed) & bit) return cudaSuccess;
+  int max_smem = 0;
+  e = cudaDeviceGetAttribute(&max_smem, cudaDevAttrMaxSharedMemoryPerMultiprocessor, dev);
+  if (e != cudaSuccess) return e;
+  int pct = max_smem > 0 ? (kb * 1024 * 100 + max_smem - 1) / max_smem : 100;
+  if (pct > 100) pct = 100;
+  e = cudaFuncSetAttribute(kernel, cudaFuncAttributePreferredSharedMemoryCarveout, pct);
+  if (e == cudaSuccess) done.fetch_or(bit, std::memory_order_relaxed);
+  return e;
+}
+
 __device__ __forceinline__ void set_status(int32_t* status, int code) {
   if (status) atomicCAS(status, 0, code);
 }
@@ -162,17 +189,21 @@ struct SweepSeg {
   int32_t* counters;      // [rows]
 };
 
+// Work layouts of the sweep: each warp its own (row, chunk), or each CTA one (row, split).
+enum SweepMode { SWEEP_ROWS = 0, SWEEP_SPLIT = 1 };
+
 struct SweepLaunch {
   SweepSeg seg[2];
   int nseg;
   int V;
-  int nchunk;
+  int mode;               // SweepMode
+  int nchunk;             // chunks per row (a multiple of 4 for SWEEP_SPLIT)
   int KP;
   int dtype;              // brisk_dtype of the logits
   int32_t* status;
 };
 
-int sweep_chunks(int rows_per_tensor, int V, int dtype, int num_sms);
+int sweep_chunks(int rows_per_tensor, int V, int dtype, int mode);
 int kp_for(int K);
 cudaError_t launch_sweep(const SweepLaunch& a, cudaStream_t stream);
 
@@ -213,8 +244,6 @@ struct ScanArgs {
   int B, L, V, K, S, logits_dt;
   int select_mode, verify_mode;
   int do_select, do_verify;
-  int ubuf;              // residual-row buffers in shared memory (set by launch_scan)
-  int tcand;             // token-share rows of the candidates staged in shared memory (set by launch_scan)
   // corrector inputs
   const void* logits_q;
   const int32_t* cand_ids;

@@ -399,11 +399,13 @@ cudaError_t gemm_tc_grouped(const TcSpec* spec, int nprob, int32_t* status, cuda
   if (stages == 2) {
     cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(smem));
+    if (e == cudaSuccess) e = prefer_carveout(gemm_tc_kernel<2>, CARVEOUT_GEMM_KB);
     if (e != cudaSuccess) return e;
     gemm_tc_kernel<2><<<total, TC_THREADS, smem, stream>>>(maps[0], maps[1], maps[2], maps[3], a);
   } else {
     cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(smem));
+    if (e == cudaSuccess) e = prefer_carveout(gemm_tc_kernel<4>, CARVEOUT_GEMM_KB);
     if (e != cudaSuccess) return e;
     gemm_tc_kernel<4><<<total, TC_THREADS, smem, stream>>>(maps[0], maps[1], maps[2], maps[3], a);
   }

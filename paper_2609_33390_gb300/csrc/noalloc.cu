@@ -54,7 +54,7 @@ extern "C" brisk_status brisk_topk_candidates_noalloc(const brisk_dims* d, const
     return BRISK_ERR_INVALID_ARG;
   // scratch layout: status word, arrival counters, per-chunk partial results
   const int rows = d->B * d->L;
-  const int nchunk = sweep_chunks(rows, d->V, d->logits_dtype, 0);
+  const int nchunk = sweep_chunks(rows, d->V, d->logits_dtype, SWEEP_ROWS);
   const int KP = kp_for(d->K);
   const size_t np = (size_t)rows * nchunk;
   const size_t o_cnt = 256;
@@ -86,6 +86,7 @@ extern "C" brisk_status brisk_topk_candidates_noalloc(const brisk_dims* d, const
   s.part_s = reinterpret_cast<float*>(scratch + o_s);
   a.nseg = 1;
   a.V = d->V;
+  a.mode = SWEEP_ROWS;
   a.nchunk = nchunk;
   a.KP = KP;
   a.dtype = d->logits_dtype;

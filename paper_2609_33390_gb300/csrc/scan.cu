@@ -23,113 +23,50 @@ namespace {
 
 constexpr int SCAN_THREADS = 128;
 constexpr int SCAN_WARPS = SCAN_THREADS / 32;
-constexpr int MCH = 2;          // 4-element state chunks per thread: S <= 4 * 128 * MCH = 1024
 
 struct Smem {
-  float* s;        // [S]     state (read back by nothing in the step loop; kept for debugging layout)
-  float* F;        // [10][S] Fz then Fh, feature-major
-  float* gpart;    // [2][SCAN_WARPS] gate partial sums (double-buffered)
-  float* red;      // [2][SCAN_WARPS][32] residual-dot partial sums after the warp reduce-scatter
   int* cid;        // [L][K]
-  float* clp;      // [L][K]
-  float* top;      // [L][3]  l_i(c_0), l_i(c_1), l_i(c_3)
-  float* lprev;    // [L][K]  l_i(c_{i-1,k}); row 0 holds l_0(x0) in slot 0
   int* sel;        // [L]
   int* rank;       // [L]
   float* ref;      // [L][K]
   float* bsum;     // [nblk]  residual block sums
   float* misc;     // [16]
   int* imisc;      // [16]
-  float* U;        // [nbuf][K][S]  residual rows of a position's candidates
-  float* Tc;       // [nbuf][K][2S] token-share rows of the previous position's candidates
-  uint64_t* full;  // [nbuf] mbarriers: the bulk copies of a buffer have landed
 };
 
 __host__ __device__ inline size_t align16(size_t x) { return (x + 15) & ~size_t(15); }
 
 constexpr int RES_BLOCK = 256;  // residual-sampling block: 32 lanes x 8 ids
 
-__host__ __device__ inline size_t smem_layout(int L, int K, int S, int V, int nbuf, int tcand,
-                                              char* base, Smem* sm) {
+__host__ __device__ inline size_t smem_layout(int L, int K, int S, int V, char* base, Smem* sm) {
   size_t off = 0;
   auto take = [&](size_t bytes) {
     const size_t o = off;
     off = align16(off + bytes);
     return base ? base + o : nullptr;
   };
+  (void)S;
   const int nblk = (V + RES_BLOCK - 1) / RES_BLOCK;
-  char* p_s = take(sizeof(float) * S);
-  char* p_F = take(sizeof(float) * 10 * S);
-  char* p_g = take(sizeof(float) * 2 * SCAN_WARPS);
-  char* p_red = take(sizeof(float) * 2 * SCAN_WARPS * 32);
   char* p_cid = take(sizeof(int) * L * K);
-  char* p_clp = take(sizeof(float) * L * K);
-  char* p_top = take(sizeof(float) * L * 3);
-  char* p_lprev = take(sizeof(float) * L * K);
   char* p_sel = take(sizeof(int) * L);
   char* p_rank = take(sizeof(int) * L);
   char* p_ref = take(sizeof(float) * L * K);
   char* p_bsum = take(sizeof(float) * nblk);
   char* p_misc = take(sizeof(float) * 16);
   char* p_imisc = take(sizeof(int) * 16);
-  char* p_U = take(sizeof(float) * nbuf * K * S);
-  char* p_Tc = take(tcand ? sizeof(float) * nbuf * K * 2 * S : 0);
-  char* p_full = take(sizeof(uint64_t) * 4);
   if (sm) {
-    sm->full = (uint64_t*)p_full;
-    sm->s = (float*)p_s; sm->F = (float*)p_F; sm->gpart = (float*)p_g; sm->red = (float*)p_red;
-    sm->cid = (int*)p_cid; sm->clp = (float*)p_clp; sm->top = (float*)p_top;
-    sm->lprev = (float*)p_lprev; sm->sel = (int*)p_sel; sm->rank = (int*)p_rank;
-    sm->ref = (float*)p_ref; sm->bsum = (float*)p_bsum; sm->misc = (float*)p_misc;
-    sm->imisc = (int*)p_imisc; sm->U = (float*)p_U; sm->Tc = (float*)p_Tc;
+    sm->cid = (int*)p_cid; sm->sel = (int*)p_sel; sm->rank = (int*)p_rank; sm->ref = (float*)p_ref;
+    sm->bsum = (float*)p_bsum; sm->misc = (float*)p_misc; sm->imisc = (int*)p_imisc;
   }
   return off;
 }
 
 __device__ __forceinline__ float4 ld4(const float* p) { return *reinterpret_cast<const float4*>(p); }
-__device__ __forceinline__ void prefetch_l2(const void* p) {
-  asm volatile("prefetch.global.L2 [%0];" ::"l"(p));
+// Cached in L2 only: rows read once per step must not displace the L1 lines that hold a
+// concurrent streaming kernel's loads in flight.
+__device__ __forceinline__ float4 ldcg4(const float* p) {
+  return __ldcg(reinterpret_cast<const float4*>(p));
 }
-__device__ __forceinline__ uint32_t su32(const void* p) {
-  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
-__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
-  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(su32(bar)), "r"(count) : "memory");
-}
-__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
-  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(su32(bar)), "r"(bytes)
-               : "memory");
-}
-__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
-  uint32_t ok;
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-      "selp.u32 %0, 1, 0, p;\n\t}"
-      : "=r"(ok)
-      : "r"(su32(bar)), "r"(parity)
-      : "memory");
-  return ok != 0;
-}
-constexpr long long SCAN_WAIT_LIMIT_CYCLES = 4000000000ll;   // about 2 s of SM clock
-// Bounded wait for a phase of an mbarrier; false when it expired.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
-  if (mbar_try_wait(bar, parity)) return true;
-  const long long t0 = clock64();
-  for (unsigned n = 1;; ++n) {
-    if (mbar_try_wait(bar, parity)) return true;
-    if ((n & 63) == 0 && clock64() - t0 > SCAN_WAIT_LIMIT_CYCLES) return false;
-  }
-}
-// Bulk (TMA) copy of `bytes` (a multiple of 16, 16-byte aligned ends) completing on `bar`.
-__device__ __forceinline__ void bulk_copy(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
-  asm volatile(
-      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
-          su32(dst)),
-      "l"(src), "r"(bytes), "r"(su32(bar))
-      : "memory");
-}
-
 // Logistic function with the hardware exponential (relative error ~1e-6).
 __device__ __forceinline__ float sigmoid_fast(float x) { return __fdividef(1.f, 1.f + __expf(-x)); }
 
@@ -156,11 +93,6 @@ __device__ __forceinline__ float reduce_scatter(float (&v)[NP]) {
 __device__ __forceinline__ float load_logit(const void* base, int dt, size_t idx) {
   if (dt == BRISK_DT_BF16) return __bfloat162float(reinterpret_cast<const __nv_bfloat16*>(base)[idx]);
   return reinterpret_cast<const float*>(base)[idx];
-}
-
-// Residual dot d_k of one position: the four warps' partial sums, added in a fixed order.
-__device__ __forceinline__ float dot_k(const float* red, int k) {
-  return ((red[k] + red[32 + k]) + red[64 + k]) + red[96 + k];
 }
 
 // Select with lane k holding refined score k (lanes >= K hold -inf); the same in every lane.
@@ -409,81 +341,242 @@ __device__ void verify_sequence(const ScanArgs& a, const Smem& sm, int b) {
     a.out_tokens[(size_t)b * L + t] = t < j ? sm.sel[t] : (t == j ? corr : -1);
 }
 
-// The sequential corrector over the positions of sequence b (Algorithm 1(b) loop). Thread t owns
-// the 4-element state chunks c = t + 128 m: it updates them, stages its own chunks of the
-// candidates' residual and token-share rows with cp.async (nbuf - 1 positions ahead; no other
-// thread reads them, so its own wait suffices), and contributes its partial residual dots, which
-// one warp reduce-scatter and one block barrier per position turn into the K dots.
+// Verification of one sequence per CTA (Sec. 3.1; Sec. 3.3; App. B Eq. 8), reading the
+// selections and refined scores the corrector wrote.
+__global__ void __launch_bounds__(SCAN_THREADS)
+verify_kernel(const __grid_constant__ ScanArgs a) {
+  extern __shared__ __align__(16) char smem_raw[];
+  Smem sm;
+  smem_layout(a.L, a.K, a.S, a.V, smem_raw, &sm);
+  const int b = blockIdx.x;
+  const int tid = threadIdx.x;
+  const int L = a.L, K = a.K, V = a.V;
+  const size_t bL = (size_t)b * L;
+  // Ids are gathered with below, so out-of-range ones (a row with no finite logit leaves
+  // placeholder ids; caller-provided ids may be anything) are replaced by 0 and reported.
+  for (int e = tid; e < L * K; e += SCAN_THREADS) {
+    int c = a.cand_ids[bL * K + e];
+    if (c < 0 || c >= V) { set_status(a.status, BRISK_ERR_NUMERIC); c = 0; }
+    sm.cid[e] = c;
+    sm.ref[e] = a.refined[bL * K + e];
+  }
+  for (int e = tid; e < L; e += SCAN_THREADS) {
+    int x = a.sel_tokens[bL + e];
+    if (x < 0 || x >= V) { set_status(a.status, BRISK_ERR_INVALID_ARG); x = 0; }
+    sm.sel[e] = x;
+  }
+  __syncthreads();
+  // each selection's rank in its candidate list
+  for (int i = tid; i < L; i += SCAN_THREADS) {
+    int r = 0;
+    for (int k = 0; k < K; ++k)
+      if (sm.cid[i * K + k] == sm.sel[i]) { r = k; break; }
+    sm.rank[i] = r;
+  }
+  __syncthreads();
+  verify_sequence(a, sm, b);
+}
+
+// ---------------------------------------------------------------- corrector
+// The sequential corrector (Sec. 3.3 Eqs. 4-5; App. C.2 Eq. 7; Algorithm 1(b) loop), one CTA of
+// NW warps per sequence. Lane l of warp w owns the 4-element state chunks
+// c = l + 32 (w + NW m), m < CMC. A position's step needs no block barrier when NW = 1: the
+// residual dots and the gate are reduced with warp shuffles, and Select runs on lane k =
+// candidate k. Candidate rows are read through L2 (prefetched two positions ahead); only small
+// per-sequence tables live in shared memory, so the kernel leaves most of every SM to the
+// verifier-row sweep that runs beside it.
+constexpr int CMC = 4;
+
+struct CorrSmem {
+  float* F;      // [2][S][5]  Fz then Fh
+  float* wg;     // [S]
+  int* cid;      // [L][K]
+  float* clp;    // [L][K]
+  float* top;    // [L][3]  l_i(c_0), l_i(c_1), l_i(c_3)
+  float* lprev;  // [L][K]  l_i(c_{i-1,k}); row 0 holds l_0(x0) in slot 0
+  float* red;    // [2][NW][32] per-warp reduced residual dots (NW > 1)
+  float* gpart;  // [2][NW]
+};
+
+__host__ __device__ inline size_t corr_layout(int L, int K, int S, int NW, char* base,
+                                              CorrSmem* sm) {
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    const size_t o = off;
+    off = align16(off + bytes);
+    return base ? base + o : nullptr;
+  };
+  char* pF = take(sizeof(float) * 10 * S);
+  char* pw = take(sizeof(float) * S);
+  char* pc = take(sizeof(int) * L * K);
+  char* pl = take(sizeof(float) * L * K);
+  char* pt = take(sizeof(float) * L * 3);
+  char* pp = take(sizeof(float) * L * K);
+  char* pr = take(sizeof(float) * 2 * NW * 32);
+  char* pg = take(sizeof(float) * 2 * NW);
+  if (sm) {
+    sm->F = (float*)pF; sm->wg = (float*)pw;
+    sm->cid = (int*)pc; sm->clp = (float*)pl; sm->top = (float*)pt; sm->lprev = (float*)pp;
+    sm->red = (float*)pr; sm->gpart = (float*)pg;
+  }
+  return off;
+}
+
+// Brings the K rows of `row_floats` floats at table + ids[k] * row_floats into L2 without
+// waiting: one 128-byte line per lane and instruction. (Line prefetches disturb a concurrent
+// streaming kernel far less than bulk prefetches of whole rows.)
+__device__ __forceinline__ void prefetch_rows_l2(const float* table, const int* ids, int K,
+                                                 int row_floats) {
+  const int lane = threadIdx.x & 31;
+  const int lines = row_floats / 32;
+  for (int k = 0; k < K; ++k) {
+    const float* row = table + (size_t)ids[k] * row_floats;
+    for (int l = lane; l < lines; l += 32) asm volatile("prefetch.global.L2 [%0];" ::"l"(row + 32 * l));
+  }
+}
+
+// Warp reduce-scatter of NP values per lane (NP = 8, 16 or 32): afterwards lane l holds the
+// warp-wide sum of value (l >> log2(32 / NP)) & (NP - 1), that is value k sits in lane
+// k * (32 / NP).
 template <int NP>
-__device__ void corrector_loop(const ScanArgs& a, const Smem& sm, int b, int x0) {
+__device__ __forceinline__ float reduce_scatter_n(float (&v)[NP]) {
+  const int lane = threadIdx.x & 31;
+#pragma unroll
+  for (int m = 16, n = NP; n > 1; m >>= 1, n >>= 1) {
+    const bool upper = (lane & m) != 0;
+#pragma unroll
+    for (int j = 0; j < n / 2; ++j) {
+      const float send = upper ? v[j] : v[j + n / 2];
+      const float keep = upper ? v[j + n / 2] : v[j];
+      v[j] = keep + __shfl_xor_sync(FULL_MASK, send, m);
+    }
+  }
+  float r = v[0];
+#pragma unroll
+  for (int m = 32 / NP / 2; m >= 1; m >>= 1) r += __shfl_xor_sync(FULL_MASK, r, m);
+  return r;
+}
+
+// Gathers logits at nidx (row, column) pairs into dst, eight loads in flight per lane.
+template <int NT, typename IndexOf>
+__device__ __forceinline__ void gather_logits(const void* logits, int dt, int n, float* dst,
+                                              IndexOf index_of) {
+  const int tid = threadIdx.x;
+  for (int base = 0; base < n; base += 8 * NT) {
+    float v[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const int e = base + j * NT + tid;
+      v[j] = e < n ? load_logit(logits, dt, index_of(e)) : 0.f;
+    }
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const int e = base + j * NT + tid;
+      if (e < n) dst[e] = v[j];
+    }
+  }
+}
+
+// The sequential corrector (Sec. 3.3 Eqs. 4-5; App. C.2 Eq. 7; Algorithm 1(b) loop), one CTA of
+// NW warps per sequence. Lane l of warp w owns the 4-element state chunks
+// c = l + 32 (w + NW m), m < CMC. A position's step needs no block barrier when NW = 1: the
+// residual dots and the gate are reduced with warp shuffles, and Select runs with lane k holding
+// candidate k. Every load of the step is issued unconditionally (chunk and candidate indices
+// clamped into range, the surplus contributions multiplied by zero state or never read) so the
+// compiler can keep them all in flight. Candidate rows are read through L2, prefetched two
+// positions ahead; shared memory holds only small per-sequence tables, so the kernel leaves most
+// of every SM to the verifier-row sweep that runs beside it.
+template <int NW, int NP>
+__global__ void __launch_bounds__(NW * 32)
+corrector_kernel(const __grid_constant__ ScanArgs a) {
+  extern __shared__ __align__(16) char smem_raw[];
+  CorrSmem sm;
+  corr_layout(a.L, a.K, a.S, NW, smem_raw, &sm);
+  constexpr int NT = NW * 32;
+  constexpr int LSTEP = 32 / NP;           // lane stride between reduced dots
+  const int b = blockIdx.x;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int L = a.L, K = a.K, S = a.S;
+  const int L = a.L, K = a.K, S = a.S, V = a.V;
   const size_t bL = (size_t)b * L;
   const int nch = S / 4;
-  const int nbuf = a.ubuf, tcand = a.tcand;
 
-  float4 s4[MCH], wg4[MCH], gz4[MCH], gh4[MCH], tz4[MCH], th4[MCH];
+  for (int e = tid; e < L * K; e += NT) {
+    int c = a.cand_ids[bL * K + e];
+    if (c < 0 || c >= V) { set_status(a.status, BRISK_ERR_NUMERIC); c = 0; }
+    sm.cid[e] = c;
+    sm.clp[e] = a.cand_logprob[bL * K + e];
+  }
+  int x0 = a.x0[b];
+  if (x0 < 0 || x0 >= V) {
+    if (tid == 0) set_status(a.status, BRISK_ERR_INVALID_ARG);
+    x0 = 0;
+  }
+  // the feature shares and the gate weights, read every step, into shared memory
+  for (int e = tid; e < 5 * S / 4; e += NT) {
+    reinterpret_cast<float4*>(sm.F)[e] = ld4(a.Fz + 4 * e);
+    reinterpret_cast<float4*>(sm.F + 5 * S)[e] = ld4(a.Fh + 4 * e);
+  }
+  for (int e = tid; e < S / 4; e += NT) reinterpret_cast<float4*>(sm.wg)[e] = ld4(a.wg + 4 * e);
+  __syncthreads();
+  // into L2: the first two positions' residual rows, and the token-share row of the first
+  // position's rank-0 candidate (the usual next previous token; others are fetched on demand,
+  // since speculative rows for every rank would cost the concurrent sweep far more DRAM
+  // bandwidth than the rare miss costs here)
+  if (warp == 0) {
+    prefetch_rows_l2(a.U, sm.cid, K * (L > 1 ? 2 : 1), S);
+    if (L > 1) prefetch_rows_l2(a.Tzh, sm.cid, 1, 2 * S);
+  }
+  // the features' logit gathers, all independent of the selections
+  const void* lq = a.logits_q;
+  const int ldt = a.logits_dt;
+  gather_logits<NT>(lq, ldt, L * 3, sm.top, [&](int e) {
+    const int i = e / 3, w = e % 3;
+    return (bL + i) * V + sm.cid[i * K + (w == 0 ? 0 : (w == 1 ? 1 : 3))];
+  });
+  gather_logits<NT>(lq, ldt, L * K, sm.lprev, [&](int e) {
+    const int i = e / K, k = e % K;
+    return i == 0 ? bL * V + x0 : (bL + i) * V + sm.cid[(i - 1) * K + k];
+  });
+
+  // lane chunks, clamped into range; a chunk past the state keeps s = 0 throughout
+  int cc[CMC];
+  bool ok[CMC];
 #pragma unroll
-  for (int m = 0; m < MCH; ++m) {
-    const int c = tid + m * SCAN_THREADS;
-    s4[m] = wg4[m] = gz4[m] = gh4[m] = tz4[m] = th4[m] = make_float4(0.f, 0.f, 0.f, 0.f);
-    if (c < nch) {
-      const float4 g0 = ld4(a.G0 + (size_t)b * S + 4 * c), t0 = ld4(a.T0 + (size_t)x0 * S + 4 * c);
-      s4[m] = make_float4(tanhf(g0.x + t0.x), tanhf(g0.y + t0.y), tanhf(g0.z + t0.z),
-                          tanhf(g0.w + t0.w));                     // s_{-1} = u_0 = Init(h_c, E(x0))
-      wg4[m] = ld4(a.wg + 4 * c);
-      gz4[m] = ld4(a.G + bL * 2 * S + 4 * c);
-      gh4[m] = ld4(a.G + bL * 2 * S + S + 4 * c);
-      tz4[m] = ld4(a.Tzh + (size_t)x0 * 2 * S + 4 * c);           // token share of x_{-1} = x0
-      th4[m] = ld4(a.Tzh + (size_t)x0 * 2 * S + S + 4 * c);
-    }
+  for (int m = 0; m < CMC; ++m) {
+    const int c = lane + 32 * (warp + NW * m);
+    ok[m] = c < nch;
+    cc[m] = ok[m] ? c : nch - 1;
+  }
+  float4 s4[CMC], gz4[CMC], gh4[CMC], tz4[CMC], th4[CMC];
+#pragma unroll
+  for (int m = 0; m < CMC; ++m) {
+    const int c = cc[m];
+    const float4 g0 = ldcg4(a.G0 + (size_t)b * S + 4 * c), t0 = ldcg4(a.T0 + (size_t)x0 * S + 4 * c);
+    s4[m] = ok[m] ? make_float4(tanhf(g0.x + t0.x), tanhf(g0.y + t0.y), tanhf(g0.z + t0.z),
+                                tanhf(g0.w + t0.w))        // s_{-1} = u_0 = Init(h_c, E(x0))
+                  : make_float4(0.f, 0.f, 0.f, 0.f);
+    gz4[m] = ldcg4(a.G + bL * 2 * S + 4 * c);
+    gh4[m] = ldcg4(a.G + bL * 2 * S + S + 4 * c);
+    tz4[m] = ldcg4(a.Tzh + (size_t)x0 * 2 * S + 4 * c);   // token share of x_{-1} = x0
+    th4[m] = ldcg4(a.Tzh + (size_t)x0 * 2 * S + S + 4 * c);
   }
   float wgf[5];
 #pragma unroll
   for (int f = 0; f < 5; ++f) wgf[f] = a.wg[S + f];
   const float sig_alpha = sigmoidf_(a.alpha);
-
-  // The rows position j needs (the residual rows of its candidates and, when staged, the
-  // token-share rows of the previous position's candidates) arrive in buffer j % nbuf by bulk
-  // copies that thread 0 issues; everybody waits on that buffer's mbarrier.
-  const uint32_t u_bytes = (uint32_t)S * 4, t_bytes = (uint32_t)S * 8;
-  auto issue = [&](int j) {
-    if (tid != 0 || j >= L) return;
-    const int slot = j % nbuf;
-    float* Ub = sm.U + (size_t)slot * K * S;
-    float* Tb = sm.Tc + (size_t)slot * K * 2 * S;
-    const bool with_t = tcand && j > 0;
-    mbar_expect_tx(&sm.full[slot], K * (u_bytes + (with_t ? t_bytes : 0)));
-    for (int k = 0; k < K; ++k) {
-      bulk_copy(Ub + (size_t)k * S, a.U + (size_t)sm.cid[j * K + k] * S, u_bytes, &sm.full[slot]);
-      if (with_t)
-        bulk_copy(Tb + (size_t)k * 2 * S, a.Tzh + (size_t)sm.cid[(j - 1) * K + k] * 2 * S, t_bytes,
-                  &sm.full[slot]);
-    }
-  };
-  if (tid == 0) {
-    for (int q = 0; q < nbuf; ++q) mbar_init(&sm.full[q], 1);
-    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-  }
   __syncthreads();
-  const int ahead = nbuf > 1 ? nbuf - 1 : 0;
-  for (int j = 0; j < (nbuf > 1 ? ahead : 1); ++j) issue(j);
-  // this thread's share of the L2 prefetch of a table row: fixed across positions
-  const int u_lines = (S * 4 + 127) / 128, t_lines = (S * 8 + 127) / 128;
-  const int pu_k = tid / u_lines, pu_l = tid % u_lines;
-  bool timed_out = false;
 
   int prev = x0, prank = 0;
   float u_cur = (a.select_mode == BRISK_SELECT_SAMPLE) ? a.u_sel[bL] : 0.f;
   for (int i = 0; i < L; ++i) {
     const int buf = i & 1;
     const int* ci = sm.cid + i * K;
-    if (nbuf > 1) issue(i + ahead);
-    // L2 prefetch further ahead (and of the gathered token-share rows when they are not staged)
-    if (i + nbuf < L && pu_k < K) prefetch_l2(a.U + (size_t)ci[nbuf * K + pu_k] * S + pu_l * 32);
-    if (!tcand && i + 1 < L)
-      for (int e = tid; e < K * t_lines; e += SCAN_THREADS)
-        prefetch_l2(a.Tzh + (size_t)ci[e / t_lines] * 2 * S + (e % t_lines) * 32);
+    // into L2, for step i + 2: its residual rows, and the token-share row of the next
+    // position's rank-0 candidate
+    if (warp == 0 && i + 2 < L) {
+      prefetch_rows_l2(a.U, ci + 2 * K, K, S);
+      prefetch_rows_l2(a.Tzh, ci + K, 1, 2 * S);
+    }
     // confidence features of position i (App. C.2)
     const float l0 = sm.top[i * 3 + 0];
     float phi[5];
@@ -492,214 +585,138 @@ __device__ void corrector_loop(const ScanArgs& a, const Smem& sm, int b, int x0)
     phi[2] = (prev == ci[0]) ? 1.f : 0.f;
     phi[3] = (prev == ci[0] || prev == ci[1] || prev == ci[2] || prev == ci[3]) ? 1.f : 0.f;
     phi[4] = l0 - sm.lprev[i * K + (i == 0 ? 0 : prank)];
-    // the rows of position i have landed
-    if (!mbar_wait(&sm.full[i % nbuf], (i / nbuf) & 1)) timed_out = true;
-    const float* Ub = sm.U + (size_t)(i % nbuf) * K * S;
     // token share of the previous token (x0's came with the prologue)
     if (i > 0) {
-      const float* Tp = tcand ? sm.Tc + ((size_t)(i % nbuf) * K + prank) * 2 * S
-                              : a.Tzh + (size_t)prev * 2 * S;
+      const float* Tp = a.Tzh + (size_t)prev * 2 * S;
 #pragma unroll
-      for (int m = 0; m < MCH; ++m) {
-        const int c = tid + m * SCAN_THREADS;
-        if (c < nch) {
-          tz4[m] = ld4(Tp + 4 * c);
-          th4[m] = ld4(Tp + S + 4 * c);
-        }
+      for (int m = 0; m < CMC; ++m) {
+        tz4[m] = ldcg4(Tp + 4 * cc[m]);
+        th4[m] = ldcg4(Tp + S + 4 * cc[m]);
       }
     }
-    // minimal-GRU step on this thread's chunks, its gate partial and its residual-dot partials
+    // minimal-GRU step on this lane's chunks and its gate partial
     float gacc = 0.f;
-    float part[NP];
 #pragma unroll
-    for (int k = 0; k < NP; ++k) part[k] = 0.f;
+    for (int m = 0; m < CMC; ++m) {
+      const int c = cc[m];
+      float zp[4] = {gz4[m].x + tz4[m].x, gz4[m].y + tz4[m].y, gz4[m].z + tz4[m].z,
+                     gz4[m].w + tz4[m].w};
+      float hp[4] = {gh4[m].x + th4[m].x, gh4[m].y + th4[m].y, gh4[m].z + th4[m].z,
+                     gh4[m].w + th4[m].w};
+      // feature shares of this chunk's four elements: 20 contiguous floats of F[S, 5]
+      float fz[20], fh[20];
 #pragma unroll
-    for (int m = 0; m < MCH; ++m) {
-      const int c = tid + m * SCAN_THREADS;
-      if (c < nch) {
-        float zp[4] = {gz4[m].x + tz4[m].x, gz4[m].y + tz4[m].y, gz4[m].z + tz4[m].z,
-                       gz4[m].w + tz4[m].w};
-        float hp[4] = {gh4[m].x + th4[m].x, gh4[m].y + th4[m].y, gh4[m].z + th4[m].z,
-                       gh4[m].w + th4[m].w};
+      for (int q = 0; q < 5; ++q) {
+        const float4 vz = ld4(sm.F + 20 * c + 4 * q);
+        const float4 vh = ld4(sm.F + 5 * S + 20 * c + 4 * q);
+        fz[4 * q] = vz.x; fz[4 * q + 1] = vz.y; fz[4 * q + 2] = vz.z; fz[4 * q + 3] = vz.w;
+        fh[4 * q] = vh.x; fh[4 * q + 1] = vh.y; fh[4 * q + 2] = vh.z; fh[4 * q + 3] = vh.w;
+      }
+#pragma unroll
+      for (int e = 0; e < 4; ++e)
 #pragma unroll
         for (int f = 0; f < 5; ++f) {
-          const float4 fz = ld4(sm.F + (size_t)f * S + 4 * c);
-          const float4 fh = ld4(sm.F + (size_t)(5 + f) * S + 4 * c);
-          zp[0] = fmaf(fz.x, phi[f], zp[0]); zp[1] = fmaf(fz.y, phi[f], zp[1]);
-          zp[2] = fmaf(fz.z, phi[f], zp[2]); zp[3] = fmaf(fz.w, phi[f], zp[3]);
-          hp[0] = fmaf(fh.x, phi[f], hp[0]); hp[1] = fmaf(fh.y, phi[f], hp[1]);
-          hp[2] = fmaf(fh.z, phi[f], hp[2]); hp[3] = fmaf(fh.w, phi[f], hp[3]);
+          zp[e] = fmaf(fz[5 * e + f], phi[f], zp[e]);
+          hp[e] = fmaf(fh[5 * e + f], phi[f], hp[e]);
         }
-        float sv[4] = {s4[m].x, s4[m].y, s4[m].z, s4[m].w};
+      float sv[4] = {s4[m].x, s4[m].y, s4[m].z, s4[m].w};
 #pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const float z = sigmoid_fast(zp[e]);
-          sv[e] = (1.f - z) * sv[e] + z * hp[e];
-        }
-        s4[m] = make_float4(sv[0], sv[1], sv[2], sv[3]);
-        gacc = fmaf(wg4[m].x, sv[0], gacc);
-        gacc = fmaf(wg4[m].y, sv[1], gacc);
-        gacc = fmaf(wg4[m].z, sv[2], gacc);
-        gacc = fmaf(wg4[m].w, sv[3], gacc);
-#pragma unroll
-        for (int k = 0; k < NP; ++k) {
-          if (k < K) {
-            const float4 u = ld4(Ub + (size_t)k * S + 4 * c);
-            part[k] = fmaf(u.x, sv[0], fmaf(u.y, sv[1], fmaf(u.z, sv[2], fmaf(u.w, sv[3], part[k]))));
-          }
-        }
+      for (int e = 0; e < 4; ++e) {
+        const float z = sigmoid_fast(zp[e]);
+        sv[e] = ok[m] ? (1.f - z) * sv[e] + z * hp[e] : 0.f;
       }
+      s4[m] = make_float4(sv[0], sv[1], sv[2], sv[3]);
+      const float4 w4 = ld4(sm.wg + 4 * c);
+      gacc = fmaf(w4.x, sv[0], fmaf(w4.y, sv[1], fmaf(w4.z, sv[2], fmaf(w4.w, sv[3], gacc))));
+    }
+    // residual-dot partials with the rows of this position's candidates (rank K-1 repeated
+    // past K)
+    float part[NP];
+#pragma unroll
+    for (int k = 0; k < NP; ++k) {
+      const float* Uk = a.U + (size_t)ci[k < K ? k : K - 1] * S;
+      float acc = 0.f;
+#pragma unroll
+      for (int m = 0; m < CMC; ++m) {
+        const float4 u = ldcg4(Uk + 4 * cc[m]);
+        acc = fmaf(u.x, s4[m].x, fmaf(u.y, s4[m].y, fmaf(u.z, s4[m].z, fmaf(u.w, s4[m].w, acc))));
+      }
+      part[k] = acc;
     }
     // hidden and position shares of the next position: plain loads first used in the next step
     if (i + 1 < L) {
       const float* Gn = a.G + (bL + i + 1) * 2 * S;
 #pragma unroll
-      for (int m = 0; m < MCH; ++m) {
-        const int c = tid + m * SCAN_THREADS;
-        if (c < nch) {
-          gz4[m] = ld4(Gn + 4 * c);
-          gh4[m] = ld4(Gn + S + 4 * c);
-        }
+      for (int m = 0; m < CMC; ++m) {
+        gz4[m] = ldcg4(Gn + 4 * cc[m]);
+        gh4[m] = ldcg4(Gn + S + 4 * cc[m]);
       }
     }
-    // block reduction: residual dots by one reduce-scatter per warp, gate partial by a warp sum
-    const float r = reduce_scatter<NP>(part);
-    const int v = NP == 16 ? ((lane >> 1) & 15) : lane;
-    float* red = sm.red + buf * SCAN_WARPS * 32;
-    if (v < K && (NP == 32 || (lane & 1) == 0)) red[warp * 32 + v] = r;
+    // residual dots by a warp reduce-scatter; across warps through shared memory
+    float r = reduce_scatter_n<NP>(part);
     gacc = warp_sum(gacc);
-    if (lane == 0) sm.gpart[buf * SCAN_WARPS + warp] = gacc;
-    __syncthreads();
-    if (nbuf == 1) issue(i + 1);   // every thread is done with the single buffer
+    if (NW > 1) {
+      float* red = sm.red + buf * NW * 32;
+      if ((lane & (LSTEP - 1)) == 0) red[warp * 32 + lane / LSTEP] = r;
+      if (lane == 0) sm.gpart[buf * NW + warp] = gacc;
+      __syncthreads();
+      const int vidx = (lane / LSTEP) & (NP - 1);
+      r = red[vidx];
+      gacc = sm.gpart[buf * NW];
+      for (int w = 1; w < NW; ++w) {
+        r += red[w * 32 + vidx];
+        gacc += sm.gpart[buf * NW + w];
+      }
+    }
     // gate, refined scores (lane k: candidate k) and Select, identically in every warp
-    float gate = a.b_g;
-    for (int w = 0; w < SCAN_WARPS; ++w) gate += sm.gpart[buf * SCAN_WARPS + w];
+    float gate = a.b_g + gacc;
 #pragma unroll
     for (int f = 0; f < 5; ++f) gate = fmaf(wgf[f], phi[f], gate);
     const float gamma = sig_alpha * sigmoid_fast(gate);
-    const float* clp = sm.clp + i * K;
-    const float ref = lane < K ? clp[lane] + gamma * dot_k(red, lane) : -INFINITY;
+    const float dk = __shfl_sync(FULL_MASK, r, (lane * LSTEP) & 31);
+    const float ref = lane < K ? sm.clp[i * K + lane] + gamma * dk : -INFINITY;
     const int pick = select_warp(ref, K, a.select_mode, u_cur);
-    if (warp == 0 && lane < K) {
-      sm.ref[i * K + lane] = ref;
-      a.refined[(bL + i) * K + lane] = ref;
-    }
+    if (warp == 0 && lane < K) a.refined[(bL + i) * K + lane] = ref;
     if (a.select_mode == BRISK_SELECT_SAMPLE && i + 1 < L) u_cur = a.u_sel[bL + i + 1];
     prank = pick;
     prev = ci[pick];
-    if (tid == 0) {
-      sm.sel[i] = prev;
-      sm.rank[i] = pick;
-      a.sel_tokens[bL + i] = prev;
-    }
+    if (tid == 0) a.sel_tokens[bL + i] = prev;
   }
-  if (timed_out && lane == 0) set_status(a.status, BRISK_ERR_TIMEOUT);
-  // every copy that was issued has been waited for above (the last one at position L - 1)
-}
-
-__global__ void __launch_bounds__(SCAN_THREADS)
-scan_kernel(const __grid_constant__ ScanArgs a) {
-  extern __shared__ __align__(16) char smem_raw[];
-  Smem sm;
-  smem_layout(a.L, a.K, a.S, a.V, a.ubuf, a.tcand, smem_raw, &sm);
-  const int b = blockIdx.x;
-  const int tid = threadIdx.x;
-  const int L = a.L, K = a.K, S = a.S, V = a.V;
-  const size_t bL = (size_t)b * L;
-
-  // Ids are gathered with below, so out-of-range ones (a row with no finite logit leaves
-  // placeholder ids; caller-provided ids may be anything) are replaced by 0 and reported.
-  for (int e = tid; e < L * K; e += SCAN_THREADS) {
-    int c = a.cand_ids[bL * K + e];
-    if (c < 0 || c >= V) { set_status(a.status, BRISK_ERR_NUMERIC); c = 0; }
-    sm.cid[e] = c;
-  }
-  if (a.do_select) {
-    for (int e = tid; e < L * K; e += SCAN_THREADS) sm.clp[e] = a.cand_logprob[bL * K + e];
-  } else {
-    for (int e = tid; e < L * K; e += SCAN_THREADS) sm.ref[e] = a.refined[bL * K + e];
-    for (int e = tid; e < L; e += SCAN_THREADS) {
-      int x = a.sel_tokens[bL + e];
-      if (x < 0 || x >= V) { set_status(a.status, BRISK_ERR_INVALID_ARG); x = 0; }
-      sm.sel[e] = x;
-    }
-  }
-  __syncthreads();
-
-  if (a.do_select) {
-    int x0 = a.x0[b];
-    if (x0 < 0 || x0 >= V) {
-      if (tid == 0) set_status(a.status, BRISK_ERR_INVALID_ARG);
-      x0 = 0;
-    }
-    // features' logit gathers, all independent of the selections
-    for (int e = tid; e < L * 3; e += SCAN_THREADS) {
-      const int i = e / 3, w = e % 3;
-      const int c = sm.cid[i * K + (w == 0 ? 0 : (w == 1 ? 1 : 3))];
-      sm.top[e] = load_logit(a.logits_q, a.logits_dt, (bL + i) * V + c);
-    }
-    for (int e = tid; e < L * K; e += SCAN_THREADS) {
-      const int i = e / K, k = e % K;
-      float v = 0.f;
-      if (i == 0) { if (k == 0) v = load_logit(a.logits_q, a.logits_dt, bL * V + x0); }
-      else v = load_logit(a.logits_q, a.logits_dt, (bL + i) * V + sm.cid[(i - 1) * K + k]);
-      sm.lprev[e] = v;
-    }
-    for (int e = tid; e < 5 * S; e += SCAN_THREADS) {
-      const int j = e / 5, f = e % 5;
-      sm.F[f * S + j] = a.Fz[e];
-      sm.F[(5 + f) * S + j] = a.Fh[e];
-    }
-    if (K + 1 <= 16) corrector_loop<16>(a, sm, b, x0);
-    else corrector_loop<32>(a, sm, b, x0);
-    __syncthreads();
-  } else {
-    // verify alone: recover each selection's rank in its candidate list
-    for (int i = tid; i < L; i += SCAN_THREADS) {
-      int r = 0;
-      for (int k = 0; k < K; ++k)
-        if (sm.cid[i * K + k] == sm.sel[i]) { r = k; break; }
-      sm.rank[i] = r;
-    }
-    __syncthreads();
-  }
-
-  if (a.do_verify) verify_sequence(a, sm, b);
 }
 
 }  // namespace
 
-constexpr size_t SCAN_SMEM_LIMIT = 227 * 1024;
-
-// Shared-memory plan: stage the token-share rows and prefetch two positions ahead when that
-// fits, else less.
-void scan_plan(int L, int K, int S, int V, int* nbuf, int* tcand) {
-  const int plans[5][2] = {{3, 1}, {2, 1}, {3, 0}, {2, 0}, {1, 0}};
-  for (const auto& p : plans) {
-    if (smem_layout(L, K, S, V, p[0], p[1], nullptr, nullptr) <= SCAN_SMEM_LIMIT) {
-      *nbuf = p[0];
-      *tcand = p[1];
-      return;
-    }
-  }
-  *nbuf = 1;
-  *tcand = 0;
-}
-
 size_t scan_smem_bytes(int L, int K, int S, int V) {
-  int ubuf, tcand;
-  scan_plan(L, K, S, V, &ubuf, &tcand);
-  return smem_layout(L, K, S, V, ubuf, tcand, nullptr, nullptr);
+  return smem_layout(L, K, S, V, nullptr, nullptr);
 }
 
-cudaError_t launch_scan(const ScanArgs& a_in, cudaStream_t stream) {
-  ScanArgs a = a_in;
-  scan_plan(a.L, a.K, a.S, a.V, &a.ubuf, &a.tcand);
-  const size_t smem = smem_layout(a.L, a.K, a.S, a.V, a.ubuf, a.tcand, nullptr, nullptr);
-  cudaError_t e = cudaFuncSetAttribute(scan_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       (int)smem);
+template <int NW, int NP>
+cudaError_t launch_corrector(const ScanArgs& a, cudaStream_t stream) {
+  const size_t smem = corr_layout(a.L, a.K, a.S, NW, nullptr, nullptr);
+  cudaError_t e = cudaFuncSetAttribute(corrector_kernel<NW, NP>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e == cudaSuccess) e = prefer_carveout(corrector_kernel<NW, NP>, CARVEOUT_SMALL_KB);
   if (e != cudaSuccess) return e;
-  scan_kernel<<<a.B, SCAN_THREADS, smem, stream>>>(a);
+  corrector_kernel<NW, NP><<<a.B, NW * 32, smem, stream>>>(a);
+  return cudaGetLastError();
+}
+
+// The corrector (do_select) or the verification (do_verify) for every sequence.
+cudaError_t launch_scan(const ScanArgs& a, cudaStream_t stream) {
+  if (a.do_select) {
+    if (a.S > 4 * 32 * CMC) {
+      if (a.K <= 8) return launch_corrector<2, 8>(a, stream);
+      return a.K <= 16 ? launch_corrector<2, 16>(a, stream) : launch_corrector<2, 32>(a, stream);
+    }
+    if (a.K <= 8) return launch_corrector<1, 8>(a, stream);
+    return a.K <= 16 ? launch_corrector<1, 16>(a, stream) : launch_corrector<1, 32>(a, stream);
+  }
+  const size_t smem = scan_smem_bytes(a.L, a.K, a.S, a.V);
+  cudaError_t e = cudaFuncSetAttribute(verify_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)smem);
+  if (e == cudaSuccess) e = prefer_carveout(verify_kernel, CARVEOUT_SMALL_KB);
+  if (e != cudaSuccess) return e;
+  verify_kernel<<<a.B, SCAN_THREADS, smem, stream>>>(a);
   return cudaGetLastError();
 }
 

@@ -10,20 +10,24 @@
 // so far: a 16-byte vector whose max is below T cannot contribute, so the
 // common case costs one compare per vector. The rare vectors that reach T are
 // broadcast to the whole warp and their elements inserted cooperatively.
-// When a row is split into several chunks, each warp writes its partial
-// result to the workspace and the last warp to finish the row (arrival
-// counter, no waiting) merges the partials in chunk order, so results do not
-// depend on timing.
+// The warps of a CTA either sweep different rows or split one row (the two
+// layouts of sweep_kernel). Partial results of one row are merged in chunk
+// order, in shared memory within a CTA and otherwise through the workspace
+// by the last warp to finish the row (arrival counter, no waiting), so
+// results do not depend on timing.
 #include "brisk_internal.cuh"
 
 namespace brisk {
 
 namespace {
 
-constexpr int SWEEP_WARPS = 4;                 // independent warps per CTA
+constexpr int SWEEP_WARPS = 4;                 // warps of a split-layout CTA (and the most)
+constexpr int SWEEP_ROW_WARPS = 2;             // warps of a row-layout CTA: small CTAs pack
+                                               // around a concurrent kernel's CTAs
 constexpr int SWEEP_UNROLL = 8;                // 16-byte loads in flight per lane
 constexpr int SWEEP_TARGET_TASKS = 152 * 16;   // warp tasks per tensor the chunking aims for
 constexpr int SWEEP_MIN_VEC_PER_LANE = 32;
+constexpr int SWEEP_CHUNK_VEC = 4096;          // 16-byte vectors a split-layout chunk (64 KB)
 
 // Online log-sum-exp of one group of N logits whose max is mx.
 template <int N>
@@ -83,37 +87,30 @@ __device__ __forceinline__ float warp_kth_largest(float x, int k) {
   return __shfl_sync(FULL_MASK, x, 32 - k);
 }
 
-// The rare path. Every lane of the warp has stashed its SWEEP_UNROLL vectors in shared memory;
-// vector u of lane l holds ids id0(l) + u * 32 * VN + j. Each vector whose max reaches T is read
-// by the whole warp (a broadcast from shared memory) and its elements at or above T are
-// inserted in id order. Kept out of the unrolled main loop: one copy of the insertion code.
+// The rare path, for one vector slot u in which some lane's vector reaches T. Every lane has
+// written its vector u to the warp's buffer in shared memory; vector u of lane l holds ids
+// id0(l) + u * 32 * VN + j. Each vector whose max (mx, per lane) reaches T is read by the whole
+// warp (a broadcast from shared memory) and its elements at or above T are inserted in id
+// order. Kept out of the unrolled main loop: one copy of the insertion code.
 template <typename T>
-__device__ __forceinline__ void offer_stash(const uint4* warp_stash, unsigned umask, int id0_lane,
-                                         float& thr, float& wv, int& wi, int kout) {
+__device__ __noinline__ void offer_vector(const uint4* warp_buf, float mx, int id0_lane, int u,
+                                          float& thr, float& wv, int& wi, int kout) {
   constexpr int VN = Vec<T>::N;
   const int lane = threadIdx.x & 31;
-#pragma unroll 1
-  while (umask) {   // only the vector slots u where some lane reached the threshold
-    const int u = __ffs(umask) - 1;
-    umask &= umask - 1;
-    float f[VN];
-    unpack(warp_stash[lane * SWEEP_UNROLL + u], f, T());
-    unsigned trig = __ballot_sync(FULL_MASK, max_of(f) >= thr);
-    while (trig) {
-      const int src = __ffs(trig) - 1;
-      trig &= trig - 1;
-      // lane j < VN reads element j of lane src's vector; the ones at or above T are inserted
-      // in id order
-      const T* e = reinterpret_cast<const T*>(warp_stash + src * SWEEP_UNROLL + u);
-      const float g = lane < VN ? to_f32(e[lane]) : -INFINITY;
-      const int id0 = __shfl_sync(FULL_MASK, id0_lane, src) + u * 32 * VN;
-      unsigned em = __ballot_sync(FULL_MASK, lane < VN && g >= thr);
-      while (em) {
-        const int j = __ffs(em) - 1;
-        em &= em - 1;
-        const float gj = __shfl_sync(FULL_MASK, g, j);
-        if (gj >= thr) thr = fmaxf(thr, wlist_insert(gj, id0 + j, wv, wi, kout));
-      }
+  unsigned trig = __ballot_sync(FULL_MASK, mx >= thr);
+  while (trig) {
+    const int src = __ffs(trig) - 1;
+    trig &= trig - 1;
+    // lane j < VN reads element j of lane src's vector
+    const T* e = reinterpret_cast<const T*>(warp_buf + src);
+    const float g = lane < VN ? to_f32(e[lane]) : -INFINITY;
+    const int id0 = __shfl_sync(FULL_MASK, id0_lane, src) + u * 32 * VN;
+    unsigned em = __ballot_sync(FULL_MASK, lane < VN && g >= thr);
+    while (em) {
+      const int j = __ffs(em) - 1;
+      em &= em - 1;
+      const float gj = __shfl_sync(FULL_MASK, g, j);
+      if (gj >= thr) thr = fmaxf(thr, wlist_insert(gj, id0 + j, wv, wi, kout));
     }
   }
 }
@@ -156,39 +153,27 @@ __device__ __forceinline__ void finalize_row(const SweepSeg& sg, int row, float 
   if (lane == 0) sg.out_lse[row] = lse;
 }
 
+// One warp's sweep of chunk `chunk` (of nchunk) of the row at rowp: on return every lane holds
+// the chunk's (max, sum of exp) pair and the warp list holds its best-first top-kout.
 template <typename T>
-__global__ void __launch_bounds__(SWEEP_WARPS * 32)
-sweep_kernel(const __grid_constant__ SweepLaunch a) {
+__device__ __forceinline__ void sweep_chunk(const T* rowp, int V, int chunk, int nchunk, int kout,
+                                            uint4* warp_buf, float& m, float& s, float& wv,
+                                            int& wi) {
   constexpr int VN = Vec<T>::N;
-  __shared__ uint4 stash[SWEEP_WARPS * 32 * SWEEP_UNROLL];
-  const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  uint4* warp_stash = stash + warp * 32 * SWEEP_UNROLL;
-  const long long task = (long long)blockIdx.x * SWEEP_WARPS + warp;
-  const long long tasks0 = (long long)a.seg[0].rows * a.nchunk;
-  const long long total = tasks0 + (a.nseg > 1 ? (long long)a.seg[1].rows * a.nchunk : 0);
-  if (task >= total) return;
-  const int si = task < tasks0 ? 0 : 1;
-  const SweepSeg& sg = a.seg[si];
-  const long long t = si ? task - tasks0 : task;
-  const int row = (int)(t / a.nchunk);
-  const int chunk = (int)(t % a.nchunk);
-  const int V = a.V;
-  const int kout = sg.kout;
-
-  const T* rowp = reinterpret_cast<const T*>(sg.logits) + (size_t)row * V;
   const uintptr_t addr = reinterpret_cast<uintptr_t>(rowp);
   int head = (int)(((16u - (unsigned)(addr & 15u)) & 15u) / sizeof(T));
   if (head > V) head = V;
   const int nvec = (V - head) / VN;
   const int tail0 = head + nvec * VN;
-  const int vpc = (nvec + a.nchunk - 1) / a.nchunk;
+  const int vpc = (nvec + nchunk - 1) / nchunk;
   const int v_begin = chunk * vpc;
   const int v_end = min(nvec, v_begin + vpc);
 
-  float m = -INFINITY, s = 0.f;        // this lane's running max and sum of exp(x - max)
-  float wv = -INFINITY;                // warp list entry held by this lane
-  int wi = INVALID_ID;
+  m = -INFINITY;                       // this lane's running max and sum of exp(x - max)
+  s = 0.f;
+  wv = -INFINITY;                      // warp list entry held by this lane
+  wi = INVALID_ID;
   float thr = -INFINITY;               // warp-uniform lower bound on the K-th best so far
 
   // unaligned head (ids below every vector): lanes 0..head-1 of chunk 0
@@ -237,14 +222,18 @@ sweep_kernel(const __grid_constant__ SweepLaunch a) {
     umask = __reduce_or_sync(FULL_MASK, umask);
     if (umask) {
 #pragma unroll
-      for (int u = 0; u < SWEEP_UNROLL; ++u) warp_stash[lane * SWEEP_UNROLL + u] = w[u];
-      __syncwarp();
-      offer_stash<T>(warp_stash, umask, head + (base + lane) * VN, thr, wv, wi, kout);
-      __syncwarp();
+      for (int u = 0; u < SWEEP_UNROLL; ++u) {
+        if (umask & (1u << u)) {
+          warp_buf[lane] = w[u];
+          __syncwarp();
+          offer_vector<T>(warp_buf, mx[u], head + (base + lane) * VN, u, thr, wv, wi, kout);
+          __syncwarp();
+        }
+      }
     }
   }
   // ragged tail (ids above every vector): lanes of the last chunk, one element each
-  if (chunk == a.nchunk - 1) {
+  if (chunk == nchunk - 1) {
     const int e = tail0 + lane;
     float f = -INFINITY;
     if (e < V) {
@@ -254,19 +243,21 @@ sweep_kernel(const __grid_constant__ SweepLaunch a) {
     }
     offer_scalars(f, e < V ? e : INVALID_ID, thr, wv, wi, kout);
   }
-
   warp_lse_combine(m, s);
-  const float ov = wv;
-  const int oi = wi;
-  if (a.nchunk == 1) {
-    finalize_row(sg, row, m, s, ov, oi, a.status);
-    return;
-  }
+}
 
-  const size_t pb = (size_t)row * a.nchunk + chunk;
+// Publishes one partial result (part index pb of the row) and, in the last of the row's
+// `parts` warps to arrive (arrival counter, no waiting), merges all of them in part order and
+// writes the row's outputs. Called by one whole warp.
+__device__ __forceinline__ void publish_partial(const SweepSeg& sg, int row, int pb_in_row,
+                                                int parts, int KP, float m, float s, float wv,
+                                                int wi, int32_t* status) {
+  const int lane = threadIdx.x & 31;
+  const int kout = sg.kout;
+  const size_t pb = (size_t)row * parts + pb_in_row;
   if (lane < kout) {
-    sg.part_val[pb * a.KP + lane] = ov;
-    sg.part_id[pb * a.KP + lane] = oi;
+    sg.part_val[pb * KP + lane] = wv;
+    sg.part_id[pb * KP + lane] = wi;
   }
   if (lane == 0) {
     sg.part_m[pb] = m;
@@ -277,15 +268,15 @@ sweep_kernel(const __grid_constant__ SweepLaunch a) {
   int prev = 0;
   if (lane == 0) prev = atomicAdd(&sg.counters[row], 1);
   prev = __shfl_sync(FULL_MASK, prev, 0);
-  if (prev != a.nchunk - 1) return;
+  if (prev != parts - 1) return;
   __threadfence();
 
-  // last warp of the row: merge the chunk partials in chunk order
+  // last part of the row: merge the partials in part order
   wv = -INFINITY;
   wi = INVALID_ID;
-  thr = -INFINITY;
-  for (int c = 0; c < a.nchunk; ++c) {
-    const size_t q = ((size_t)row * a.nchunk + c) * a.KP;
+  float thr = -INFINITY;
+  for (int c = 0; c < parts; ++c) {
+    const size_t q = ((size_t)row * parts + c) * KP;
     float f = -INFINITY;
     int id = INVALID_ID;
     if (lane < kout) {
@@ -295,21 +286,106 @@ sweep_kernel(const __grid_constant__ SweepLaunch a) {
     offer_scalars(f, id, thr, wv, wi, kout);
   }
   float mm = -INFINITY, ss = 0.f;
-  for (int c = lane; c < a.nchunk; c += 32) {
-    const size_t q = (size_t)row * a.nchunk + c;
+  for (int c = lane; c < parts; c += 32) {
+    const size_t q = (size_t)row * parts + c;
     lse_merge(mm, ss, __ldcg(sg.part_m + q), __ldcg(sg.part_s + q));
   }
   warp_lse_combine(mm, ss);
-  finalize_row(sg, row, mm, ss, wv, wi, a.status);
+  finalize_row(sg, row, mm, ss, wv, wi, status);
   if (lane == 0) sg.counters[row] = 0;
+}
+
+// Two work layouts (SweepLaunch::mode):
+//  SWEEP_ROWS : each warp sweeps its own (row, chunk) task; a CTA holds blockDim / 32 tasks.
+//               One warp sees a whole row when the row is not split, so the top-K threshold
+//               tightens over the whole row (the proposal rows' layout).
+//  SWEEP_SPLIT: a CTA sweeps one (row, split): its warps take consecutive chunks and merge in
+//               shared memory. Many short CTAs let the block scheduler balance the work over
+//               SMs that a concurrent kernel slows down (the verifier rows' layout, which runs
+//               beside the corrector).
+// At most 64 registers a thread: eight 4-warp CTAs fit an SM's register file, so a full wave
+// of the sweep still fits beside a CTA of a concurrent kernel.
+template <typename T, int MODE>
+__global__ void __launch_bounds__(SWEEP_WARPS * 32, 8)
+sweep_kernel(const __grid_constant__ SweepLaunch a) {
+  __shared__ uint4 stash[SWEEP_WARPS * 32];
+  __shared__ float mvals[SWEEP_WARPS][32];
+  __shared__ int mids[SWEEP_WARPS][32];
+  __shared__ float mms[SWEEP_WARPS][2];
+  const int nw = blockDim.x >> 5;
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  uint4* warp_buf = stash + warp * 32;
+  const int V = a.V;
+
+  if constexpr (MODE == SWEEP_ROWS) {
+    const long long task = (long long)blockIdx.x * nw + warp;
+    const long long tasks0 = (long long)a.seg[0].rows * a.nchunk;
+    const long long total = tasks0 + (a.nseg > 1 ? (long long)a.seg[1].rows * a.nchunk : 0);
+    if (task >= total) return;
+    const int si = task < tasks0 ? 0 : 1;
+    const SweepSeg& sg = a.seg[si];
+    const long long t = si ? task - tasks0 : task;
+    const int row = (int)(t / a.nchunk);
+    const int chunk = (int)(t % a.nchunk);
+    const T* rowp = reinterpret_cast<const T*>(sg.logits) + (size_t)row * V;
+    float m, s, wv;
+    int wi;
+    sweep_chunk<T>(rowp, V, chunk, a.nchunk, sg.kout, warp_buf, m, s, wv, wi);
+    if (a.nchunk == 1) finalize_row(sg, row, m, s, wv, wi, a.status);
+    else publish_partial(sg, row, chunk, a.nchunk, a.KP, m, s, wv, wi, a.status);
+    return;
+  } else {
+
+  const int nsplit = a.nchunk / nw;                     // CTAs per row
+  const long long ctas0 = (long long)a.seg[0].rows * nsplit;
+  const long long cta = blockIdx.x;
+  const int si = cta < ctas0 ? 0 : 1;
+  const SweepSeg& sg = a.seg[si];
+  const long long t = si ? cta - ctas0 : cta;
+  const int row = (int)(t / nsplit);
+  const int split = (int)(t % nsplit);
+  const int kout = sg.kout;
+  const T* rowp = reinterpret_cast<const T*>(sg.logits) + (size_t)row * V;
+  float m, s, wv;
+  int wi;
+  sweep_chunk<T>(rowp, V, split * nw + warp, a.nchunk, kout, warp_buf, m, s, wv, wi);
+  // the CTA's warps merged by warp 0 in chunk order
+  mvals[warp][lane] = wv;
+  mids[warp][lane] = wi;
+  if (lane == 0) {
+    mms[warp][0] = m;
+    mms[warp][1] = s;
+  }
+  __syncthreads();
+  if (warp != 0) return;
+  float thr = -INFINITY;
+  for (int w = 1; w < nw; ++w) {
+    offer_scalars(lane < kout ? mvals[w][lane] : -INFINITY, lane < kout ? mids[w][lane] : INVALID_ID,
+                  thr, wv, wi, kout);
+    lse_merge(m, s, mms[w][0], mms[w][1]);
+  }
+  if (nsplit == 1) finalize_row(sg, row, m, s, wv, wi, a.status);
+  else publish_partial(sg, row, split, nsplit, a.KP, m, s, wv, wi, a.status);
+  }
 }
 
 template <typename T>
 cudaError_t launch_t(const SweepLaunch& a, cudaStream_t stream) {
-  long long tasks = (long long)a.seg[0].rows * a.nchunk;
-  if (a.nseg > 1) tasks += (long long)a.seg[1].rows * a.nchunk;
-  const unsigned grid = (unsigned)((tasks + SWEEP_WARPS - 1) / SWEEP_WARPS);
-  sweep_kernel<T><<<grid, SWEEP_WARPS * 32, 0, stream>>>(a);
+  long long rows = a.seg[0].rows;
+  if (a.nseg > 1) rows += a.seg[1].rows;
+  if (a.mode == SWEEP_ROWS) {
+    const long long tasks = rows * a.nchunk;
+    const unsigned grid = (unsigned)((tasks + SWEEP_ROW_WARPS - 1) / SWEEP_ROW_WARPS);
+    const cudaError_t e = prefer_carveout(sweep_kernel<T, SWEEP_ROWS>, CARVEOUT_SMALL_KB);
+    if (e != cudaSuccess) return e;
+    sweep_kernel<T, SWEEP_ROWS><<<grid, SWEEP_ROW_WARPS * 32, 0, stream>>>(a);
+  } else {
+    const unsigned grid = (unsigned)(rows * (a.nchunk / SWEEP_WARPS));
+    const cudaError_t e = prefer_carveout(sweep_kernel<T, SWEEP_SPLIT>, CARVEOUT_SMALL_KB);
+    if (e != cudaSuccess) return e;
+    sweep_kernel<T, SWEEP_SPLIT><<<grid, SWEEP_WARPS * 32, 0, stream>>>(a);
+  }
   return cudaGetLastError();
 }
 
@@ -321,18 +397,33 @@ int kp_for(int K) {
   return kp;
 }
 
-// Chunks per row: enough warp tasks per tensor to keep every SM streaming, but at least
-// SWEEP_MIN_VEC_PER_LANE 16-byte vectors per lane. Independent of the device so that the
-// summation order, and hence every rounded result, is the same on every run.
-int sweep_chunks(int rows_per_tensor, int V, int dtype, int /*num_sms*/) {
+// Chunks per row. Independent of the device so that the summation order, and hence every
+// rounded result, is the same on every run.
+//  SWEEP_ROWS : enough warp tasks per tensor to keep every SM streaming, but at least
+//               SWEEP_MIN_VEC_PER_LANE 16-byte vectors per lane.
+//  SWEEP_SPLIT: a multiple of SWEEP_WARPS, about SWEEP_CHUNK_VEC vectors a chunk, and enough
+//               CTAs per tensor to keep every SM streaming.
+int sweep_chunks(int rows_per_tensor, int V, int dtype, int mode) {
   const int vn = dtype == BRISK_DT_BF16 ? 8 : 4;
   const long long nvec = V / vn;
-  long long maxc = nvec / (32LL * SWEEP_MIN_VEC_PER_LANE);
-  if (maxc < 1) maxc = 1;
-  long long c = (SWEEP_TARGET_TASKS + rows_per_tensor - 1) / rows_per_tensor;
+  if (mode == SWEEP_ROWS) {
+    long long maxc = nvec / (32LL * SWEEP_MIN_VEC_PER_LANE);
+    if (maxc < 1) maxc = 1;
+    long long c = (SWEEP_TARGET_TASKS + rows_per_tensor - 1) / rows_per_tensor;
+    if (c < 1) c = 1;
+    if (c > maxc) c = maxc;
+    return (int)c;
+  }
+  long long maxs = nvec / (32LL * SWEEP_MIN_VEC_PER_LANE * SWEEP_WARPS);
+  if (maxs < 1) maxs = 1;
+  const long long target = (SWEEP_TARGET_TASKS + SWEEP_WARPS - 1) / SWEEP_WARPS;
+  long long c = (target + rows_per_tensor - 1) / rows_per_tensor;
+  const long long per_cta = (long long)SWEEP_CHUNK_VEC * SWEEP_WARPS;
+  const long long by_size = (nvec + per_cta - 1) / per_cta;
+  if (c < by_size) c = by_size;
   if (c < 1) c = 1;
-  if (c > maxc) c = maxc;
-  return (int)c;
+  if (c > maxs) c = maxs;
+  return (int)c * SWEEP_WARPS;
 }
 
 cudaError_t launch_sweep(const SweepLaunch& a, cudaStream_t stream) {
