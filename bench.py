@@ -156,7 +156,7 @@ class ClockSampler:
 
 # ----------------------------------------------------------------------------- CPU oracle leg
 
-CPU_SAMPLE_SEQS = 8
+CPU_SAMPLE_SEQS = 24
 
 
 def _oracle_sample_worker(spec_json: str) -> str:
