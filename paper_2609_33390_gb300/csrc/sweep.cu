@@ -153,6 +153,89 @@ __device__ __forceinline__ void finalize_row(const SweepSeg& sg, int row, float 
   if (lane == 0) sg.out_lse[row] = lse;
 }
 
+// Max of the VN logits of one 16-byte vector (bf16 pairs compared packed: 3 instructions).
+__device__ __forceinline__ float vec_max(const uint4& w, __nv_bfloat16) {
+  const __nv_bfloat162 a = __hmax2(*reinterpret_cast<const __nv_bfloat162*>(&w.x),
+                                   *reinterpret_cast<const __nv_bfloat162*>(&w.y));
+  const __nv_bfloat162 b = __hmax2(*reinterpret_cast<const __nv_bfloat162*>(&w.z),
+                                   *reinterpret_cast<const __nv_bfloat162*>(&w.w));
+  const __nv_bfloat162 c = __hmax2(a, b);
+  return fmaxf(__low2float(c), __high2float(c));
+}
+__device__ __forceinline__ float vec_max(const uint4& w, float) {
+  return fmaxf(fmaxf(__uint_as_float(w.x), __uint_as_float(w.y)),
+               fmaxf(__uint_as_float(w.z), __uint_as_float(w.w)));
+}
+
+// Per-lane state of a chunk sweep.
+struct ChunkState {
+  float m, s;      // running max and sum of exp(x - max)
+  float wv;        // warp list entry held by this lane
+  int wi;
+  float thr;       // warp-uniform lower bound on the K-th best so far
+  bool first;
+};
+
+// One iteration: SWEEP_UNROLL vectors per lane, lane's vector u holding ids
+// head + (base + lane + 32 u) * VN + j. The running max moves once per iteration, so all of the
+// iteration's exponentials share one offset; arguments and sums use packed fp32 pairs.
+template <typename T>
+__device__ __forceinline__ void sweep_iteration(const uint4 (&w)[SWEEP_UNROLL], int id0_lane,
+                                                int kout, uint4* warp_buf, ChunkState& st) {
+  constexpr int VN = Vec<T>::N;
+  float mx[SWEEP_UNROLL];
+  float mx_all = -INFINITY;
+#pragma unroll
+  for (int u = 0; u < SWEEP_UNROLL; ++u) {
+    mx[u] = vec_max(w[u], T());
+    mx_all = fmaxf(mx_all, mx[u]);
+  }
+  if (mx_all > st.m) {
+    st.s *= ex2((st.m - mx_all) * LOG2E);
+    st.m = mx_all;
+  }
+  if (st.m != -INFINITY) {
+    const float nmb = -st.m * LOG2E;
+    const float2 l2e = make_float2(LOG2E, LOG2E), off = make_float2(nmb, nmb);
+    float2 acc0 = make_float2(0.f, 0.f), acc1 = make_float2(0.f, 0.f);
+#pragma unroll
+    for (int u = 0; u < SWEEP_UNROLL; ++u) {
+      float f[VN];
+      unpack(w[u], f, T());
+#pragma unroll
+      for (int j = 0; j < VN; j += 2) {
+        const float2 arg = __ffma2_rn(make_float2(f[j], f[j + 1]), l2e, off);
+        const float2 e = make_float2(ex2(arg.x), ex2(arg.y));
+        if ((j / 2 + u) & 1) acc1 = __fadd2_rn(acc1, e);
+        else acc0 = __fadd2_rn(acc0, e);
+      }
+    }
+    const float2 acc = __fadd2_rn(acc0, acc1);
+    st.s += acc.x + acc.y;
+  }
+  if (st.first) {
+    // K lanes each hold an element at least this large: a lower bound on the K-th best
+    st.thr = fmaxf(st.thr, warp_kth_largest(mx_all, kout));
+    st.first = false;
+  }
+  unsigned umask = 0;
+#pragma unroll
+  for (int u = 0; u < SWEEP_UNROLL; ++u) umask |= (mx[u] >= st.thr ? 1u : 0u) << u;
+  umask = __reduce_or_sync(FULL_MASK, umask);
+  if (umask) {
+    const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int u = 0; u < SWEEP_UNROLL; ++u) {
+      if (umask & (1u << u)) {
+        warp_buf[lane] = w[u];
+        __syncwarp();
+        offer_vector<T>(warp_buf, mx[u], id0_lane, u, st.thr, st.wv, st.wi, kout);
+        __syncwarp();
+      }
+    }
+  }
+}
+
 // One warp's sweep of chunk `chunk` (of nchunk) of the row at rowp: on return every lane holds
 // the chunk's (max, sum of exp) pair and the warp list holds its best-first top-kout.
 template <typename T>
@@ -160,6 +243,7 @@ __device__ __forceinline__ void sweep_chunk(const T* rowp, int V, int chunk, int
                                             uint4* warp_buf, float& m, float& s, float& wv,
                                             int& wi) {
   constexpr int VN = Vec<T>::N;
+  constexpr int STEP = 32 * SWEEP_UNROLL;
   const int lane = threadIdx.x & 31;
   const uintptr_t addr = reinterpret_cast<uintptr_t>(rowp);
   int head = (int)(((16u - (unsigned)(addr & 15u)) & 15u) / sizeof(T));
@@ -170,11 +254,7 @@ __device__ __forceinline__ void sweep_chunk(const T* rowp, int V, int chunk, int
   const int v_begin = chunk * vpc;
   const int v_end = min(nvec, v_begin + vpc);
 
-  m = -INFINITY;                       // this lane's running max and sum of exp(x - max)
-  s = 0.f;
-  wv = -INFINITY;                      // warp list entry held by this lane
-  wi = INVALID_ID;
-  float thr = -INFINITY;               // warp-uniform lower bound on the K-th best so far
+  ChunkState st{-INFINITY, 0.f, -INFINITY, INVALID_ID, -INFINITY, true};
 
   // unaligned head (ids below every vector): lanes 0..head-1 of chunk 0
   if (chunk == 0) {
@@ -182,55 +262,29 @@ __device__ __forceinline__ void sweep_chunk(const T* rowp, int V, int chunk, int
     if (lane < head) {
       f = to_f32(rowp[lane]);
       const float ff[1] = {f};
-      lse_update<1>(ff, f, m, s);
+      lse_update<1>(ff, f, st.m, st.s);
     }
-    offer_scalars(f, lane < head ? lane : INVALID_ID, thr, wv, wi, kout);
+    offer_scalars(f, lane < head ? lane : INVALID_ID, st.thr, st.wv, st.wi, kout);
   }
   const uint4* vp = reinterpret_cast<const uint4*>(rowp + head);
-  bool first = true;
-  for (int base = v_begin; base < v_end; base += 32 * SWEEP_UNROLL) {
+  int base = v_begin;
+  // full iterations: no bounds checks
+  for (; base + STEP <= v_end; base += STEP) {
+    uint4 w[SWEEP_UNROLL];
+#pragma unroll
+    for (int u = 0; u < SWEEP_UNROLL; ++u) w[u] = ld_stream_v4(vp + base + lane + 32 * u);
+    sweep_iteration<T>(w, head + (base + lane) * VN, kout, warp_buf, st);
+  }
+  // the ragged last iteration, padded with -inf
+  if (base < v_end) {
+    const uint32_t ninf = VN == 8 ? 0xff80ff80u : 0xff800000u;
     uint4 w[SWEEP_UNROLL];
 #pragma unroll
     for (int u = 0; u < SWEEP_UNROLL; ++u) {
       const int v = base + lane + 32 * u;
-      if (v < v_end) w[u] = ld_stream_v4(vp + v);
-      else w[u] = make_uint4(0xff80ff80u, 0xff80ff80u, 0xff80ff80u, 0xff80ff80u);  // -inf
+      w[u] = v < v_end ? ld_stream_v4(vp + v) : make_uint4(ninf, ninf, ninf, ninf);
     }
-    if constexpr (VN == 4) {
-#pragma unroll
-      for (int u = 0; u < SWEEP_UNROLL; ++u)
-        if (base + lane + 32 * u >= v_end) w[u] = make_uint4(0xff800000u, 0xff800000u, 0xff800000u, 0xff800000u);
-    }
-    float mx[SWEEP_UNROLL];
-    float mx_all = -INFINITY;
-#pragma unroll
-    for (int u = 0; u < SWEEP_UNROLL; ++u) {
-      float f[VN];
-      unpack(w[u], f, T());
-      mx[u] = max_of(f);
-      lse_update<VN>(f, mx[u], m, s);
-      mx_all = fmaxf(mx_all, mx[u]);
-    }
-    if (first) {
-      // K lanes each hold an element at least this large: a lower bound on the K-th best
-      thr = fmaxf(thr, warp_kth_largest(mx_all, kout));
-      first = false;
-    }
-    unsigned umask = 0;
-#pragma unroll
-    for (int u = 0; u < SWEEP_UNROLL; ++u) umask |= (mx[u] >= thr ? 1u : 0u) << u;
-    umask = __reduce_or_sync(FULL_MASK, umask);
-    if (umask) {
-#pragma unroll
-      for (int u = 0; u < SWEEP_UNROLL; ++u) {
-        if (umask & (1u << u)) {
-          warp_buf[lane] = w[u];
-          __syncwarp();
-          offer_vector<T>(warp_buf, mx[u], head + (base + lane) * VN, u, thr, wv, wi, kout);
-          __syncwarp();
-        }
-      }
-    }
+    sweep_iteration<T>(w, head + (base + lane) * VN, kout, warp_buf, st);
   }
   // ragged tail (ids above every vector): lanes of the last chunk, one element each
   if (chunk == nchunk - 1) {
@@ -239,11 +293,15 @@ __device__ __forceinline__ void sweep_chunk(const T* rowp, int V, int chunk, int
     if (e < V) {
       f = to_f32(rowp[e]);
       const float ff[1] = {f};
-      lse_update<1>(ff, f, m, s);
+      lse_update<1>(ff, f, st.m, st.s);
     }
-    offer_scalars(f, e < V ? e : INVALID_ID, thr, wv, wi, kout);
+    offer_scalars(f, e < V ? e : INVALID_ID, st.thr, st.wv, st.wi, kout);
   }
-  warp_lse_combine(m, s);
+  warp_lse_combine(st.m, st.s);
+  m = st.m;
+  s = st.s;
+  wv = st.wv;
+  wi = st.wi;
 }
 
 // Publishes one partial result (part index pb of the row) and, in the last of the row's
