@@ -69,7 +69,7 @@ WsLayout ws_layout(const brisk_dims* d) {
 // U   [V, S] : residual rows, U(v) = W_s^T W_c E_out(v)
 // T0  [V, S] : token share of Init, W0[:, r:2r] P_e E_in(v)
 // Tin, Tout [V, r]: P_e E_in(v), W_c E_out(v) (intermediates of the folds)
-// posG [L, 2S]: position shares W_z[:, 2r:2r+16] pos_i | W_h[:, 2r:2r+16] pos_i (added to G)
+// posG [L, 2S]: position shares W_z[:, 2r:2r+16] pos_i | W_h[:, 2r:2r+16] pos_i
 // Fz, Fh [S, 5]: feature shares W_z[:, 2r+16:] P_phi, W_h[:, 2r+16:] P_phi
 // wg [S+5] fp32 copy of w_g; W2 [2S, r] = [W_z[:, :r] ; W_h[:, :r]] and W0h [S, r] = W0[:, :r] (fp32)
 // W2s [2S, 3r], W0s [S, 3r] (bf16): the same blocks written three times along k, so that
@@ -147,9 +147,11 @@ SweepSeg make_seg(const WsLayout& w, void* ws, int seg, const void* logits, int 
 // G = Hm[:BL] [W_z[:, :r] ; W_h[:, :r]]^T and G0 = Hm[BL:] W0[:, :r]^T. With bf16 weights the
 // products run on the tensor cores: the first one writes Hm as three bf16 parts, which the
 // second one multiplies by the weight blocks written three times along k (fp32-level accuracy).
+// The first product (k = d long, few 256-wide tiles) uses 64-wide tiles and a 4-deep pipeline:
+// four times the CTAs, each streaming a quarter of the weights.
 brisk_status hidden_products(const brisk_dims* d, const brisk_params* p, const void* tables,
                              const void* hidden, const void* h_ctx, const WsLayout& w, void* ws,
-                             cudaStream_t st, int stages = 4) {
+                             cudaStream_t st) {
   const TbLayout t = tb_layout(d);
   const int BL = d->B * d->L, r = d->r, S = 2 * d->r, hd = d->hidden_dtype;
   int32_t* status = at<int32_t>(ws, w.status);
@@ -158,15 +160,15 @@ brisk_status hidden_products(const brisk_dims* d, const brisk_params* p, const v
     __nv_bfloat16* Hs = at<__nv_bfloat16>(ws, w.Hm);   // [BL + B, 3r]: hi | mid | lo
     const int r3 = 3 * r;
     const TcSpec first[2] = {
-        {BL, r, d->d, hidden, d->d, p->P_h, d->d, 1, Hs, r3, nullptr, 0},
-        {d->B, r, d->d, h_ctx, d->d, p->P_h, d->d, 1, Hs + (size_t)BL * r3, r3, nullptr, 0}};
-    BRISK_CUDA(gemm_tc_grouped(first, 2, status, st, stages));
+        {BL, r, d->d, hidden, d->d, p->P_h, d->d, 1, Hs, r3, nullptr, 0, 64},
+        {d->B, r, d->d, h_ctx, d->d, p->P_h, d->d, 1, Hs + (size_t)BL * r3, r3, nullptr, 0, 64}};
+    BRISK_CUDA(gemm_tc_grouped(first, 2, status, st, 4));
     const TcSpec second[2] = {
         {BL, 2 * S, r3, Hs, r3, at<__nv_bfloat16>(tables, t.W2s), r3, 0, at<float>(ws, w.G), 2 * S,
-         at<float>(tables, t.posG), d->L},
+         nullptr, 0, 0},
         {d->B, S, r3, Hs + (size_t)BL * r3, r3, at<__nv_bfloat16>(tables, t.W0s), r3, 0,
-         at<float>(ws, w.G0), S, nullptr, 0}};
-    BRISK_CUDA(gemm_tc_grouped(second, 2, status, st, stages));
+         at<float>(ws, w.G0), S, nullptr, 0, 0}};
+    BRISK_CUDA(gemm_tc_grouped(second, 2, status, st, 2));
     return BRISK_OK;
   }
   float* Hm = at<float>(ws, w.Hm);
@@ -174,7 +176,7 @@ brisk_status hidden_products(const brisk_dims* d, const brisk_params* p, const v
   BRISK_CUDA(gemm_simt(d->B, r, d->d, h_ctx, hd, d->d, p->P_h, hd, d->d, false,
                        Hm + (size_t)BL * r, r, st));
   BRISK_CUDA(gemm_simt(BL, 2 * S, r, Hm, BRISK_DT_F32, r, at<float>(tables, t.W2), BRISK_DT_F32, r,
-                       false, at<float>(ws, w.G), 2 * S, st, at<float>(tables, t.posG), d->L));
+                       false, at<float>(ws, w.G), 2 * S, st));
   BRISK_CUDA(gemm_simt(d->B, S, r, Hm + (size_t)BL * r, BRISK_DT_F32, r, at<float>(tables, t.W0h),
                        BRISK_DT_F32, r, false, at<float>(ws, w.G0), S, st));
   return BRISK_OK;
@@ -218,6 +220,7 @@ ScanArgs scan_args(const brisk_dims* d, const brisk_params* p, const void* table
   if (tables) {
     const TbLayout t = tb_layout(d);
     a.Tzh = at<float>(tables, t.Tzh);
+    a.posG = at<float>(tables, t.posG);
     a.U = at<float>(tables, t.U);
     a.T0 = at<float>(tables, t.T0);
     a.Fz = at<float>(tables, t.Fz);
@@ -456,7 +459,7 @@ brisk_status brisk_decode_tail(const brisk_dims* d, const brisk_params* p, const
   if (!ss) return BRISK_ERR_CUDA;
   BRISK_CUDA(cudaEventRecord(ss->ev[0], st));
   BRISK_CUDA(cudaStreamWaitEvent(ss->hi, ss->ev[0], 0));
-  s = hidden_products(d, p, tables, io->hidden, io->h_ctx, w, ws, ss->hi, 2);
+  s = hidden_products(d, p, tables, io->hidden, io->h_ctx, w, ws, ss->hi);
   if (s != BRISK_OK) return s;
   BRISK_CUDA(cudaEventRecord(ss->ev[1], ss->hi));
 

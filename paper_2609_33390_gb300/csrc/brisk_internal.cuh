@@ -229,6 +229,9 @@ struct TcSpec {
   int ldc;
   const float* bias;   // optional fp32 [bias_period, N] added to row m as bias[m % bias_period] (mode 0)
   int bias_period;
+  // Widest output tile (columns) to use, 0 for the default 256; narrower tiles give more CTAs
+  // and a smaller pipeline stage. Read from the first product of a grouped launch.
+  int max_bn;
 };
 // `stages` (2 or 4) sets the shared-memory pipeline depth: 2 leaves room on each SM for other
 // kernels running concurrently.
@@ -250,7 +253,8 @@ struct ScanArgs {
   const float* cand_logprob;
   const int32_t* x0;
   const float* u_sel;
-  const float* G;        // [B*L, 2S] hidden and position shares of the GRU pre-activations (z | h)
+  const float* G;        // [B*L, 2S] hidden shares of the GRU pre-activations (z | h)
+  const float* posG;     // [L, 2S]   position shares of the GRU pre-activations (z | h)
   const float* G0;       // [B, S]    hidden-state part of Init
   const float* Tzh;      // [V, 2S]   token part of the GRU pre-activations (z | h)
   const float* U;        // [V, S]    residual rows: d = <s, U[c]>

@@ -1,12 +1,13 @@
 // Tensor-core product C[m, n] = sum_k A[m, k] B[n, k] for bf16 A, B (both K-contiguous)
 // with fp32 accumulation, on the 5th-generation tensor cores of sm_103a.
 //
-// One CTA computes one 128 x BN tile. A TMA producer thread streams 64-wide K
-// slices of A and B into a 4-stage ring of 128-byte-swizzled shared-memory
-// buffers; one thread issues tcgen05.mma (M = 128, N = BN, K = 16) into a TMEM
-// accumulator and releases each stage with tcgen05.commit; then all four warps
-// read their 32 TMEM lanes back with tcgen05.ld and write the tile. Every
-// wait on an mbarrier is bounded (about 2 s of SM clock): on expiry the CTA records BRISK_ERR_TIMEOUT,
+// One CTA computes one 128 x BN tile. A TMA producer thread streams 64-wide K slices of A and
+// B into a ring of 128-byte-swizzled shared-memory buffers; one thread issues tcgen05.mma
+// (M = 128, N = BN, K = 16) into a TMEM accumulator and releases each stage with
+// tcgen05.commit. The epilogue reads TMEM 32 columns at a time (tcgen05.ld), stages each chunk
+// in one of several shared-memory buffers (the ring is free by then) and writes it with a TMA
+// tensor store, so that staging the next chunks overlaps the stores in flight. Every wait on
+// an mbarrier is bounded (about 2 s of SM clock): on expiry the CTA records BRISK_ERR_TIMEOUT,
 // drains what it started and frees its TMEM.
 //
 // Used for the corrector's one dense contraction (the MASK hidden states times
@@ -68,6 +69,26 @@ __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, u
       " [%0], [%1, {%3, %4}], [%2];" ::"r"(su32(dst)),
       "l"(reinterpret_cast<uint64_t>(map)), "r"(su32(bar)), "r"(x), "r"(y)
       : "memory");
+}
+// TMA tensor store of a box staged in shared memory (bulk-group completion).
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, const void* src, int x, int y) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
+          reinterpret_cast<uint64_t>(map)),
+      "r"(su32(src)), "r"(x), "r"(y)
+      : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+// Waits until at most n (0, 1 or 3) committed bulk groups still read shared memory.
+__device__ __forceinline__ void bulk_wait_read(int n) {
+  if (n >= 3) asm volatile("cp.async.bulk.wait_group.read 3;" ::: "memory");
+  else if (n == 1) asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
+  else asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
+}
+__device__ __forceinline__ void bulk_wait0() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+// Makes this thread's shared-memory writes visible to the async (TMA) proxy.
+__device__ __forceinline__ void fence_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 __device__ __forceinline__ void tmem_alloc(uint32_t* slot, uint32_t ncols) {
   asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(su32(slot)),
@@ -141,11 +162,15 @@ __host__ __device__ constexpr uint32_t idesc_bf16(int M, int N) {
 struct TcProblem {
   int M, N, K;
   int mode;         // 0: fp32 C[m*ldc + n]; 1: bf16 parts hi, mid, lo at [m*ldc + {0, N, 2N} + n]
-  int ldc;
   int mtiles, ntiles;
-  void* C;
   const float* bias;   // optional fp32 [bias_period, N], added to row m as bias[m % bias_period]
   int bias_period;
+};
+
+// Tensor maps of one launch: A and B of each problem, and the output boxes (mode 0: one fp32
+// map [M, N]; mode 1: one bf16 map [M, N] per part).
+struct TcMaps {
+  CUtensorMap a[2], b[2], c[2][3];
 };
 
 struct TcArgs {
@@ -157,11 +182,13 @@ struct TcArgs {
   int32_t* status;
 };
 
+// Staging of one 32-column output chunk: fp32 (mode 0) or three bf16 parts (mode 1).
+constexpr int TC_OUT_CHUNK_F32 = TC_BM * 32 * 4;
+constexpr int TC_OUT_CHUNK_BF16X3 = 3 * TC_BM * 32 * 2;
+
 template <int TC_STAGES>
 __global__ void __launch_bounds__(TC_THREADS, 1)
-gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__ CUtensorMap tmB0,
-               const __grid_constant__ CUtensorMap tmA1, const __grid_constant__ CUtensorMap tmB1,
-               const __grid_constant__ TcArgs a) {
+gemm_tc_kernel(const __grid_constant__ TcMaps maps, const __grid_constant__ TcArgs a) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   // 1024-byte alignment of every stage buffer (required by the 128-byte swizzle atoms)
   uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -169,7 +196,8 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__
   const int b_bytes = a.BN * TC_BK * 2;
   uint8_t* sA = base;
   uint8_t* sB = base + TC_STAGES * a_bytes;
-  uint64_t* full = reinterpret_cast<uint64_t*>(sB + TC_STAGES * b_bytes);
+  const int ring = TC_STAGES * (a_bytes + b_bytes);   // reused by the epilogue's output stages
+  uint64_t* full = reinterpret_cast<uint64_t*>(base + ring);
   uint64_t* empty = full + TC_STAGES;
   uint64_t* accum = empty + TC_STAGES;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(accum + 1);
@@ -178,8 +206,8 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int pi = (a.nprob > 1 && (int)blockIdx.x >= a.tiles0) ? 1 : 0;
   const TcProblem& P = a.p[pi];
-  const CUtensorMap* tmA = pi ? &tmA1 : &tmA0;
-  const CUtensorMap* tmB = pi ? &tmB1 : &tmB0;
+  const CUtensorMap* tmA = &maps.a[pi];
+  const CUtensorMap* tmB = &maps.b[pi];
   const int tile = (int)blockIdx.x - (pi ? a.tiles0 : 0);
   const int m0 = (tile % P.mtiles) * TC_BM, n0 = (tile / P.mtiles) * a.BN;
   const int nk = (P.K + TC_BK - 1) / TC_BK;
@@ -245,42 +273,56 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__
     }
     if (!done) *abort_flag = 1;
   }
+  // drain: the producer's loads complete on their own; wait (bounded) for the ones issued
+  if (warp == 0 && lane == 0 && *abort_flag) {
+    for (int kb = (issued > TC_STAGES ? issued - TC_STAGES : 0); kb < issued; ++kb) {
+      const long long t0 = clock64();
+      while (!mbar_try_wait(&full[kb % TC_STAGES], (kb / TC_STAGES) & 1) &&
+             clock64() - t0 < WAIT_LIMIT_CYCLES) {
+      }
+    }
+  }
   __syncthreads();
   tc_fence_after();
-  // Every warp owns TMEM lanes [32*warp, 32*warp + 32) = tile rows: each thread holds one row
-  // and writes it 32 columns at a time with 16-byte stores (a row segment per thread).
-  if (!*abort_flag) {
+  const bool ok = !*abort_flag;
+  if (!ok && threadIdx.x == 0) set_status(a.status, BRISK_ERR_TIMEOUT);
+
+  // Epilogue. Warp w holds tile rows [32w, 32w + 32) in its TMEM lanes, one row a thread. A
+  // finished 32-column chunk is staged in shared memory and written by TMA tensor stores
+  // (which clip rows and columns outside the product); chunk c uses stage buffer c % nbuf, so
+  // up to nbuf stores are in flight while the next chunks are staged.
+  if (ok) {
     const uint32_t trow = tmem + (static_cast<uint32_t>(warp * 32) << 16);
-    const int row = m0 + warp * 32 + lane;
-    const bool live = row < P.M;
-    const float* brow = (P.bias && live) ? P.bias + (size_t)(row % P.bias_period) * P.N : nullptr;
-    for (int c0 = 0; c0 < a.BN; c0 += 32) {
+    const int rt = warp * 32 + lane;                 // row within the tile
+    const int row = m0 + rt;
+    const float* brow = (P.bias && row < P.M) ? P.bias + (size_t)(row % P.bias_period) * P.N : nullptr;
+    const int chunk_bytes = P.mode == 0 ? TC_OUT_CHUNK_F32 : TC_OUT_CHUNK_BF16X3;
+    const int fit = ring / chunk_bytes;
+    const int nbuf = fit >= 4 ? 4 : (fit >= 2 ? 2 : 1);
+    for (int c = 0, ci = 0; c < a.BN; c += 32, ++ci) {
       float v[32];
-      tmem_ld32(trow + c0, v);
-      const int nb = n0 + c0;
-      if (!live || nb >= P.N) continue;
-      if (P.mode == 0) {
-        float* Cr = static_cast<float*>(P.C) + (size_t)row * P.ldc + nb;
-        if (brow) {
+      tmem_ld32(trow + c, v);
+      const int nb = n0 + c;
+      if (brow) {
 #pragma unroll
-          for (int q = 0; q < 8; ++q)
-            if (nb + 4 * q + 3 < P.N) {
-              const float4 b = __ldg(reinterpret_cast<const float4*>(brow + nb) + q);
-              v[4 * q] += b.x; v[4 * q + 1] += b.y; v[4 * q + 2] += b.z; v[4 * q + 3] += b.w;
-            }
-        }
-#pragma unroll
-        for (int q = 0; q < 8; ++q) {
+        for (int q = 0; q < 8; ++q)
           if (nb + 4 * q + 3 < P.N) {
-            reinterpret_cast<float4*>(Cr)[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+            const float4 b = __ldg(reinterpret_cast<const float4*>(brow + nb) + q);
+            v[4 * q] += b.x; v[4 * q + 1] += b.y; v[4 * q + 2] += b.z; v[4 * q + 3] += b.w;
           } else {
             for (int e = 0; e < 4; ++e)
-              if (nb + 4 * q + e < P.N) Cr[4 * q + e] = v[4 * q + e] + (brow ? brow[nb + 4 * q + e] : 0.f);
+              if (nb + 4 * q + e < P.N) v[4 * q + e] += brow[nb + 4 * q + e];
           }
-        }
+      }
+      uint8_t* stage = base + (ci % nbuf) * chunk_bytes;
+      if (threadIdx.x == 0) bulk_wait_read(nbuf - 1);   // the store that last used `stage` has read it
+      __syncthreads();
+      if (P.mode == 0) {
+        float4* st = reinterpret_cast<float4*>(stage + rt * 128);
+#pragma unroll
+        for (int q = 0; q < 8; ++q) st[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
       } else {
         // three bf16 parts, hi + mid + lo = x to about 2^-24 relative
-        __nv_bfloat16* Cr = static_cast<__nv_bfloat16*>(P.C) + (size_t)row * P.ldc + nb;
         __align__(16) __nv_bfloat16 hi[32], mid[32], lo[32];
 #pragma unroll
         for (int j = 0; j < 32; ++j) {
@@ -291,34 +333,26 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__
         }
 #pragma unroll
         for (int q = 0; q < 4; ++q) {
-          if (nb + 8 * q + 7 < P.N) {
-            reinterpret_cast<uint4*>(Cr)[q] = reinterpret_cast<const uint4*>(hi)[q];
-            reinterpret_cast<uint4*>(Cr + P.N)[q] = reinterpret_cast<const uint4*>(mid)[q];
-            reinterpret_cast<uint4*>(Cr + 2 * P.N)[q] = reinterpret_cast<const uint4*>(lo)[q];
-          } else {
-            for (int e = 0; e < 8; ++e)
-              if (nb + 8 * q + e < P.N) {
-                Cr[8 * q + e] = hi[8 * q + e];
-                Cr[P.N + 8 * q + e] = mid[8 * q + e];
-                Cr[2 * P.N + 8 * q + e] = lo[8 * q + e];
-              }
-          }
+          reinterpret_cast<uint4*>(stage + rt * 64)[q] = reinterpret_cast<const uint4*>(hi)[q];
+          reinterpret_cast<uint4*>(stage + TC_BM * 64 + rt * 64)[q] = reinterpret_cast<const uint4*>(mid)[q];
+          reinterpret_cast<uint4*>(stage + 2 * TC_BM * 64 + rt * 64)[q] = reinterpret_cast<const uint4*>(lo)[q];
         }
       }
-    }
-  } else if (lane == 0) {
-    set_status(a.status, BRISK_ERR_TIMEOUT);
-    *abort_flag = 1;
-  }
-  // drain: the producer's loads complete on their own; wait (bounded) for the ones issued
-  if (warp == 0 && lane == 0 && *abort_flag) {
-    for (int kb = (issued > TC_STAGES ? issued - TC_STAGES : 0); kb < issued; ++kb) {
-      const long long t0 = clock64();
-      while (!mbar_try_wait(&full[kb % TC_STAGES], (kb / TC_STAGES) & 1) &&
-             clock64() - t0 < WAIT_LIMIT_CYCLES) {
+      fence_async_smem();
+      __syncthreads();
+      if (threadIdx.x == 0) {
+        if (P.mode == 0) {
+          tma_store_2d(&maps.c[pi][0], stage, nb, m0);
+        } else {
+#pragma unroll
+          for (int part = 0; part < 3; ++part)
+            tma_store_2d(&maps.c[pi][part], stage + part * TC_BM * 64, nb, m0);
+        }
+        bulk_commit();
       }
     }
   }
+  if (threadIdx.x == 0) bulk_wait0();             // stores complete before the CTA ends
   tc_fence_before();
   __syncthreads();
   if (warp == 0) tmem_dealloc(tmem, a.tmem_cols);
@@ -350,6 +384,28 @@ bool make_map(CUtensorMap* map, const void* ptr, int rows, int cols, int ld, int
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// Output map: [rows, cols] of fp32 or bf16 with row stride ld (elements), boxes of 32 x 128, no
+// swizzle (the epilogue stages a chunk row-major).
+bool make_out_map(CUtensorMap* map, const void* ptr, bool f32, int rows, int cols, int ld) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  const int es = f32 ? 4 : 2;
+  if (reinterpret_cast<uintptr_t>(ptr) % 16 != 0 || ((size_t)ld * es) % 16 != 0) return false;
+  cuuint64_t dims[2] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows)};
+  cuuint64_t strides[1] = {static_cast<cuuint64_t>(ld) * es};
+  cuuint32_t box[2] = {32, static_cast<cuuint32_t>(TC_BM)};
+  cuuint32_t estr[2] = {1, 1};
+  return fn(map, f32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
+            const_cast<void*>(ptr), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+            CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+int tc_bn(int nmax) {
+  int BN = ((nmax + 15) / 16) * 16;
+  return BN > 256 ? 256 : BN;
+}
+
 }  // namespace
 
 size_t gemm_tc_smem(int BN, int stages) {
@@ -368,11 +424,11 @@ cudaError_t gemm_tc_grouped(const TcSpec* spec, int nprob, int32_t* status, cuda
   if (nprob < 1 || nprob > 2 || (stages != 2 && stages != 4)) return cudaErrorInvalidValue;
   int nmax = 0;
   for (int i = 0; i < nprob; ++i) nmax = spec[i].N > nmax ? spec[i].N : nmax;
-  int BN = ((nmax + 15) / 16) * 16;
-  if (BN > 256) BN = 256;
+  if (spec[0].max_bn >= 16 && nmax > spec[0].max_bn) nmax = spec[0].max_bn;
+  const int BN = tc_bn(nmax);
   int cols = 32;
   while (cols < BN) cols *= 2;
-  CUtensorMap maps[4];
+  TcMaps maps;
   TcArgs a{};
   a.nprob = nprob;
   a.BN = BN;
@@ -381,12 +437,21 @@ cudaError_t gemm_tc_grouped(const TcSpec* spec, int nprob, int32_t* status, cuda
   int total = 0;
   for (int i = 0; i < 2; ++i) {
     const TcSpec& q = spec[i < nprob ? i : 0];
-    if (!make_map(&maps[2 * i], q.A, q.M, q.K, q.lda, TC_BM) ||
-        !make_map(&maps[2 * i + 1], q.B, q.N, q.K, q.ldb, BN))
+    if (!make_map(&maps.a[i], q.A, q.M, q.K, q.lda, TC_BM) ||
+        !make_map(&maps.b[i], q.B, q.N, q.K, q.ldb, BN))
       return cudaErrorInvalidValue;
+    if (q.mode == 0) {
+      if (!make_out_map(&maps.c[i][0], q.C, true, q.M, q.N, q.ldc)) return cudaErrorInvalidValue;
+      maps.c[i][1] = maps.c[i][2] = maps.c[i][0];
+    } else {
+      for (int part = 0; part < 3; ++part)
+        if (!make_out_map(&maps.c[i][part], static_cast<const __nv_bfloat16*>(q.C) + (size_t)part * q.N,
+                          false, q.M, q.N, q.ldc))
+          return cudaErrorInvalidValue;
+    }
     if (i >= nprob) continue;
     TcProblem& P = a.p[i];
-    P.M = q.M; P.N = q.N; P.K = q.K; P.mode = q.mode; P.ldc = q.ldc; P.C = q.C;
+    P.M = q.M; P.N = q.N; P.K = q.K; P.mode = q.mode;
     P.bias = q.bias;
     P.bias_period = q.bias_period > 0 ? q.bias_period : 1;
     P.mtiles = (q.M + TC_BM - 1) / TC_BM;
@@ -396,26 +461,20 @@ cudaError_t gemm_tc_grouped(const TcSpec* spec, int nprob, int32_t* status, cuda
   }
   if (total == 0) return cudaSuccess;
   const size_t smem = gemm_tc_smem(BN, stages);
-  if (stages == 2) {
-    cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         static_cast<int>(smem));
-    if (e == cudaSuccess) e = prefer_carveout(gemm_tc_kernel<2>, CARVEOUT_GEMM_KB);
-    if (e != cudaSuccess) return e;
-    gemm_tc_kernel<2><<<total, TC_THREADS, smem, stream>>>(maps[0], maps[1], maps[2], maps[3], a);
-  } else {
-    cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         static_cast<int>(smem));
-    if (e == cudaSuccess) e = prefer_carveout(gemm_tc_kernel<4>, CARVEOUT_GEMM_KB);
-    if (e != cudaSuccess) return e;
-    gemm_tc_kernel<4><<<total, TC_THREADS, smem, stream>>>(maps[0], maps[1], maps[2], maps[3], a);
-  }
+  auto kernel = stages == 2 ? gemm_tc_kernel<2> : gemm_tc_kernel<4>;
+  cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       static_cast<int>(smem));
+  if (e == cudaSuccess) e = stages == 2 ? prefer_carveout(gemm_tc_kernel<2>, CARVEOUT_GEMM_KB)
+                                        : prefer_carveout(gemm_tc_kernel<4>, CARVEOUT_GEMM_KB);
+  if (e != cudaSuccess) return e;
+  kernel<<<total, TC_THREADS, smem, stream>>>(maps, a);
   return cudaGetLastError();
 }
 
 cudaError_t gemm_tc(int M, int N, int K, const void* A, int lda, const void* B, int ldb, int mode,
                     void* C, int ldc, int32_t* status, cudaStream_t stream) {
   if (M <= 0 || N <= 0) return cudaSuccess;
-  const TcSpec s{M, N, K, A, lda, B, ldb, mode, C, ldc, nullptr, 0};
+  const TcSpec s{M, N, K, A, lda, B, ldb, mode, C, ldc, nullptr, 0, 0};
   return gemm_tc_grouped(&s, 1, status, stream, 4);
 }
 

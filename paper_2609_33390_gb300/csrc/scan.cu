@@ -62,6 +62,9 @@ __host__ __device__ inline size_t smem_layout(int L, int K, int S, int V, char* 
 }
 
 __device__ __forceinline__ float4 ld4(const float* p) { return *reinterpret_cast<const float4*>(p); }
+__device__ __forceinline__ float4 add4(float4 x, float4 y) {
+  return make_float4(x.x + y.x, x.y + y.y, x.z + y.z, x.w + y.w);
+}
 // Cached in L2 only: rows read once per step must not displace the L1 lines that hold a
 // concurrent streaming kernel's loads in flight.
 __device__ __forceinline__ float4 ldcg4(const float* p) {
@@ -555,8 +558,8 @@ corrector_kernel(const __grid_constant__ ScanArgs a) {
     s4[m] = ok[m] ? make_float4(tanhf(g0.x + t0.x), tanhf(g0.y + t0.y), tanhf(g0.z + t0.z),
                                 tanhf(g0.w + t0.w))        // s_{-1} = u_0 = Init(h_c, E(x0))
                   : make_float4(0.f, 0.f, 0.f, 0.f);
-    gz4[m] = ldcg4(a.G + bL * 2 * S + 4 * c);
-    gh4[m] = ldcg4(a.G + bL * 2 * S + S + 4 * c);
+    gz4[m] = add4(ldcg4(a.G + bL * 2 * S + 4 * c), ld4(a.posG + 4 * c));
+    gh4[m] = add4(ldcg4(a.G + bL * 2 * S + S + 4 * c), ld4(a.posG + S + 4 * c));
     tz4[m] = ldcg4(a.Tzh + (size_t)x0 * 2 * S + 4 * c);   // token share of x_{-1} = x0
     th4[m] = ldcg4(a.Tzh + (size_t)x0 * 2 * S + S + 4 * c);
   }
@@ -646,10 +649,11 @@ corrector_kernel(const __grid_constant__ ScanArgs a) {
     // hidden and position shares of the next position: plain loads first used in the next step
     if (i + 1 < L) {
       const float* Gn = a.G + (bL + i + 1) * 2 * S;
+      const float* Pn = a.posG + (size_t)(i + 1) * 2 * S;
 #pragma unroll
       for (int m = 0; m < CMC; ++m) {
-        gz4[m] = ldcg4(Gn + 4 * cc[m]);
-        gh4[m] = ldcg4(Gn + S + 4 * cc[m]);
+        gz4[m] = add4(ldcg4(Gn + 4 * cc[m]), ld4(Pn + 4 * cc[m]));
+        gh4[m] = add4(ldcg4(Gn + S + 4 * cc[m]), ld4(Pn + S + 4 * cc[m]));
       }
     }
     // residual dots by a warp reduce-scatter; across warps through shared memory
