@@ -381,14 +381,7 @@ verify_kernel(const __grid_constant__ ScanArgs a) {
 }
 
 // ---------------------------------------------------------------- corrector
-// The sequential corrector (Sec. 3.3 Eqs. 4-5; App. C.2 Eq. 7; Algorithm 1(b) loop), one CTA of
-// NW warps per sequence. Lane l of warp w owns the 4-element state chunks
-// c = l + 32 (w + NW m), m < CMC. A position's step needs no block barrier when NW = 1: the
-// residual dots and the gate are reduced with warp shuffles, and Select runs on lane k =
-// candidate k. Candidate rows are read through L2 (prefetched two positions ahead); only small
-// per-sequence tables live in shared memory, so the kernel leaves most of every SM to the
-// verifier-row sweep that runs beside it.
-constexpr int CMC = 4;
+constexpr int CORR_WARPS = 4;   // warps per sequence: one per SM sub-partition
 
 struct CorrSmem {
   float* F;      // [2][S][5]  Fz then Fh
@@ -482,14 +475,16 @@ __device__ __forceinline__ void gather_logits(const void* logits, int dt, int n,
 
 // The sequential corrector (Sec. 3.3 Eqs. 4-5; App. C.2 Eq. 7; Algorithm 1(b) loop), one CTA of
 // NW warps per sequence. Lane l of warp w owns the 4-element state chunks
-// c = l + 32 (w + NW m), m < CMC. A position's step needs no block barrier when NW = 1: the
-// residual dots and the gate are reduced with warp shuffles, and Select runs with lane k holding
-// candidate k. Every load of the step is issued unconditionally (chunk and candidate indices
-// clamped into range, the surplus contributions multiplied by zero state or never read) so the
-// compiler can keep them all in flight. Candidate rows are read through L2, prefetched two
-// positions ahead; shared memory holds only small per-sequence tables, so the kernel leaves most
-// of every SM to the verifier-row sweep that runs beside it.
-template <int NW, int NP>
+// c = l + 32 (w + NW m), m < CMC. The residual dots and the gate are reduced with warp
+// shuffles, then across the warps through shared memory (one block barrier a position), and
+// Select runs in every warp with lane k holding candidate k. Spreading a sequence over the
+// SM's four sub-partitions shortens the dependent chain of a position and keeps each
+// sub-partition's share small, so the verifier-row sweep beside it keeps its issue slots.
+// Every load of the step is issued unconditionally (chunk and candidate indices clamped into
+// range, the surplus contributions multiplied by zero state or never read) so the compiler can
+// keep them all in flight. Candidate rows are read through L2, prefetched two positions ahead;
+// shared memory holds only small per-sequence tables.
+template <int NW, int NP, int CMC>
 __global__ void __launch_bounds__(NW * 32)
 corrector_kernel(const __grid_constant__ ScanArgs a) {
   extern __shared__ __align__(16) char smem_raw[];
@@ -694,26 +689,28 @@ size_t scan_smem_bytes(int L, int K, int S, int V) {
   return smem_layout(L, K, S, V, nullptr, nullptr);
 }
 
-template <int NW, int NP>
+template <int NP, int CMC>
 cudaError_t launch_corrector(const ScanArgs& a, cudaStream_t stream) {
+  constexpr int NW = CORR_WARPS;
   const size_t smem = corr_layout(a.L, a.K, a.S, NW, nullptr, nullptr);
-  cudaError_t e = cudaFuncSetAttribute(corrector_kernel<NW, NP>,
+  cudaError_t e = cudaFuncSetAttribute(corrector_kernel<NW, NP, CMC>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  if (e == cudaSuccess) e = prefer_carveout(corrector_kernel<NW, NP>, CARVEOUT_SMALL_KB);
+  if (e == cudaSuccess) e = prefer_carveout(corrector_kernel<NW, NP, CMC>, CARVEOUT_SMALL_KB);
   if (e != cudaSuccess) return e;
-  corrector_kernel<NW, NP><<<a.B, NW * 32, smem, stream>>>(a);
+  corrector_kernel<NW, NP, CMC><<<a.B, NW * 32, smem, stream>>>(a);
   return cudaGetLastError();
 }
 
 // The corrector (do_select) or the verification (do_verify) for every sequence.
 cudaError_t launch_scan(const ScanArgs& a, cudaStream_t stream) {
   if (a.do_select) {
-    if (a.S > 4 * 32 * CMC) {
-      if (a.K <= 8) return launch_corrector<2, 8>(a, stream);
-      return a.K <= 16 ? launch_corrector<2, 16>(a, stream) : launch_corrector<2, 32>(a, stream);
+    // 4-element chunks per lane: S / 4 chunks over CORR_WARPS * 32 lanes (S <= 1024)
+    if (a.S > 4 * 32 * CORR_WARPS) {
+      if (a.K <= 8) return launch_corrector<8, 2>(a, stream);
+      return a.K <= 16 ? launch_corrector<16, 2>(a, stream) : launch_corrector<32, 2>(a, stream);
     }
-    if (a.K <= 8) return launch_corrector<1, 8>(a, stream);
-    return a.K <= 16 ? launch_corrector<1, 16>(a, stream) : launch_corrector<1, 32>(a, stream);
+    if (a.K <= 8) return launch_corrector<8, 1>(a, stream);
+    return a.K <= 16 ? launch_corrector<16, 1>(a, stream) : launch_corrector<32, 1>(a, stream);
   }
   const size_t smem = scan_smem_bytes(a.L, a.K, a.S, a.V);
   cudaError_t e = cudaFuncSetAttribute(verify_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
