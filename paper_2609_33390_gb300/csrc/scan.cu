@@ -418,14 +418,14 @@ __host__ __device__ inline size_t corr_layout(int L, int K, int S, int NW, char*
   return off;
 }
 
-// Brings the K rows of `row_floats` floats at table + ids[k] * row_floats into L2 without
-// waiting: one 128-byte line per lane and instruction. (Line prefetches disturb a concurrent
-// streaming kernel far less than bulk prefetches of whole rows.)
-__device__ __forceinline__ void prefetch_rows_l2(const float* table, const int* ids, int K,
-                                                 int row_floats) {
+// Brings rows k = k0, k0 + kstep, ... < K of `row_floats` floats at table + ids[k] * row_floats
+// into L2 without waiting: one 128-byte line per lane and instruction. (Line prefetches disturb
+// a concurrent streaming kernel far less than bulk prefetches of whole rows.)
+__device__ __forceinline__ void prefetch_rows_l2(const float* table, const int* ids, int k0, int kstep,
+                                                 int K, int row_floats) {
   const int lane = threadIdx.x & 31;
   const int lines = row_floats / 32;
-  for (int k = 0; k < K; ++k) {
+  for (int k = k0; k < K; k += kstep) {
     const float* row = table + (size_t)ids[k] * row_floats;
     for (int l = lane; l < lines; l += 32) asm volatile("prefetch.global.L2 [%0];" ::"l"(row + 32 * l));
   }
@@ -520,10 +520,8 @@ corrector_kernel(const __grid_constant__ ScanArgs a) {
   // position's rank-0 candidate (the usual next previous token; others are fetched on demand,
   // since speculative rows for every rank would cost the concurrent sweep far more DRAM
   // bandwidth than the rare miss costs here)
-  if (warp == 0) {
-    prefetch_rows_l2(a.U, sm.cid, K * (L > 1 ? 2 : 1), S);
-    if (L > 1) prefetch_rows_l2(a.Tzh, sm.cid, 1, 2 * S);
-  }
+  prefetch_rows_l2(a.U, sm.cid, warp, NW, K * (L > 1 ? 2 : 1), S);
+  if (L > 1 && warp == NW - 1) prefetch_rows_l2(a.Tzh, sm.cid, 0, 1, 1, 2 * S);
   // the features' logit gathers, all independent of the selections
   const void* lq = a.logits_q;
   const int ldt = a.logits_dt;
@@ -564,6 +562,25 @@ corrector_kernel(const __grid_constant__ ScanArgs a) {
   const float sig_alpha = sigmoidf_(a.alpha);
   __syncthreads();
 
+  // Software pipeline across positions: the next position's residual rows (rank K-1 repeated
+  // past K) are loaded into registers one step ahead, and so is the token-share row of this
+  // position's rank-0 candidate, the usual next previous token.
+  // (Only while the rows fit in registers: NP * CMC <= 16 vectors a lane; wider variants load
+  // them in the step.)
+  constexpr bool PIPE = NP * CMC <= 16;
+  constexpr int PK = PIPE ? NP : 1;
+  float4 ub[PK][CMC];
+  if constexpr (PIPE) {
+#pragma unroll
+    for (int k = 0; k < NP; ++k) {
+      const float* Uk = a.U + (size_t)sm.cid[k < K ? k : K - 1] * S;
+#pragma unroll
+      for (int m = 0; m < CMC; ++m) ub[k][m] = ldcg4(Uk + 4 * cc[m]);
+    }
+  }
+  float4 tsz[CMC], tsh[CMC];                 // token share of the speculated previous token
+  int ts_id = -1;
+
   int prev = x0, prank = 0;
   float u_cur = (a.select_mode == BRISK_SELECT_SAMPLE) ? a.u_sel[bL] : 0.f;
   for (int i = 0; i < L; ++i) {
@@ -571,9 +588,27 @@ corrector_kernel(const __grid_constant__ ScanArgs a) {
     const int* ci = sm.cid + i * K;
     // into L2, for step i + 2: its residual rows, and the token-share row of the next
     // position's rank-0 candidate
-    if (warp == 0 && i + 2 < L) {
-      prefetch_rows_l2(a.U, ci + 2 * K, K, S);
-      prefetch_rows_l2(a.Tzh, ci + K, 1, 2 * S);
+    if (i + 2 < L) {
+      prefetch_rows_l2(a.U, ci + 2 * K, warp, NW, K, S);
+      if (warp == NW - 1) prefetch_rows_l2(a.Tzh, ci + K, 0, 1, 1, 2 * S);
+    }
+    // into registers, for step i + 1: its residual rows and the rank-0 token-share row
+    float4 un[PK][CMC], tnz[CMC], tnh[CMC];
+    if (i + 1 < L) {
+      if constexpr (PIPE) {
+#pragma unroll
+        for (int k = 0; k < NP; ++k) {
+          const float* Uk = a.U + (size_t)ci[K + (k < K ? k : K - 1)] * S;
+#pragma unroll
+          for (int m = 0; m < CMC; ++m) un[k][m] = ldcg4(Uk + 4 * cc[m]);
+        }
+      }
+      const float* Tn = a.Tzh + (size_t)ci[0] * 2 * S;
+#pragma unroll
+      for (int m = 0; m < CMC; ++m) {
+        tnz[m] = ldcg4(Tn + 4 * cc[m]);
+        tnh[m] = ldcg4(Tn + S + 4 * cc[m]);
+      }
     }
     // confidence features of position i (App. C.2)
     const float l0 = sm.top[i * 3 + 0];
@@ -583,13 +618,22 @@ corrector_kernel(const __grid_constant__ ScanArgs a) {
     phi[2] = (prev == ci[0]) ? 1.f : 0.f;
     phi[3] = (prev == ci[0] || prev == ci[1] || prev == ci[2] || prev == ci[3]) ? 1.f : 0.f;
     phi[4] = l0 - sm.lprev[i * K + (i == 0 ? 0 : prank)];
-    // token share of the previous token (x0's came with the prologue)
+    // token share of the previous token (x0's came with the prologue; the speculated one is
+    // already in registers)
     if (i > 0) {
-      const float* Tp = a.Tzh + (size_t)prev * 2 * S;
+      if (prev == ts_id) {
 #pragma unroll
-      for (int m = 0; m < CMC; ++m) {
-        tz4[m] = ldcg4(Tp + 4 * cc[m]);
-        th4[m] = ldcg4(Tp + S + 4 * cc[m]);
+        for (int m = 0; m < CMC; ++m) {
+          tz4[m] = tsz[m];
+          th4[m] = tsh[m];
+        }
+      } else {
+        const float* Tp = a.Tzh + (size_t)prev * 2 * S;
+#pragma unroll
+        for (int m = 0; m < CMC; ++m) {
+          tz4[m] = ldcg4(Tp + 4 * cc[m]);
+          th4[m] = ldcg4(Tp + S + 4 * cc[m]);
+        }
       }
     }
     // minimal-GRU step on this lane's chunks and its gate partial
@@ -627,8 +671,7 @@ corrector_kernel(const __grid_constant__ ScanArgs a) {
       const float4 w4 = ld4(sm.wg + 4 * c);
       gacc = fmaf(w4.x, sv[0], fmaf(w4.y, sv[1], fmaf(w4.z, sv[2], fmaf(w4.w, sv[3], gacc))));
     }
-    // residual-dot partials with the rows of this position's candidates (rank K-1 repeated
-    // past K)
+    // residual-dot partials with the rows of this position's candidates
     float part[NP];
 #pragma unroll
     for (int k = 0; k < NP; ++k) {
@@ -636,7 +679,9 @@ corrector_kernel(const __grid_constant__ ScanArgs a) {
       float acc = 0.f;
 #pragma unroll
       for (int m = 0; m < CMC; ++m) {
-        const float4 u = ldcg4(Uk + 4 * cc[m]);
+        float4 u;
+        if constexpr (PIPE) u = ub[k][m];
+        else u = ldcg4(Uk + 4 * cc[m]);
         acc = fmaf(u.x, s4[m].x, fmaf(u.y, s4[m].y, fmaf(u.z, s4[m].z, fmaf(u.w, s4[m].w, acc))));
       }
       part[k] = acc;
@@ -680,6 +725,21 @@ corrector_kernel(const __grid_constant__ ScanArgs a) {
     prank = pick;
     prev = ci[pick];
     if (tid == 0) a.sel_tokens[bL + i] = prev;
+    // advance the pipeline
+    if (i + 1 < L) {
+      if constexpr (PIPE) {
+#pragma unroll
+        for (int k = 0; k < NP; ++k)
+#pragma unroll
+          for (int m = 0; m < CMC; ++m) ub[k][m] = un[k][m];
+      }
+#pragma unroll
+      for (int m = 0; m < CMC; ++m) {
+        tsz[m] = tnz[m];
+        tsh[m] = tnh[m];
+      }
+      ts_id = ci[0];
+    }
   }
 }
 
