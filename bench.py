@@ -334,6 +334,14 @@ def run_ours(args):
     acc = sum(int(outs[s]["accepted_len"].sum()) for s in range(args.warmup, nsteps))
     committed = sum(int((outs[s]["accepted_len"] + (outs[s]["correction"] >= 0).int()).sum())
                     for s in range(args.warmup, nsteps))
+    # acceptance profile of the timed steps (Sec. 3.2 Eqs. 2-3), counted after the timed region
+    acc_counts = torch.zeros(2 * wl.L, dtype=torch.int64, device=dev)
+    for s in range(args.warmup, nsteps):
+        brisk.acceptance_counts(outs[s]["accepted_len"], wl.L, acc_counts)
+    counts_h = acc_counts.cpu().tolist()
+    reach_h, accept_h = counts_h[:wl.L], counts_h[wl.L:]
+    prof_a = [accept_h[i] / reach_h[i] if reach_h[i] else 0.0 for i in range(wl.L)]
+    prof_tpf, _, prof_w = brisk.acceptance_weights(prof_a)
     sweep_q_ms = [events[s][0].elapsed_time(events[s][1]) for s in range(args.warmup, nsteps)]
     sweep_p_ms = [events[s][2].elapsed_time(events[s][3]) for s in range(args.warmup, nsteps)]
     sweep_ms = [q + p for q, p in zip(sweep_q_ms, sweep_p_ms)]
@@ -400,6 +408,10 @@ def run_ours(args):
         "committed_tokens_per_s": committed_all / elapsed_max,
         "host_enqueue_us_per_step": 1e6 * host_enqueue_s / args.steps,
         "accepted_per_sequence_block": tokens / (wl.B * world * args.steps),
+        "acceptance_profile": {"a": [round(x, 4) for x in prof_a[:8]],
+                               "positions_shown": min(8, wl.L),
+                               "tpf_unit_cost": prof_tpf,
+                               "w_bar": [round(x, 4) for x in prof_w[:8]]},
     }
     print(json.dumps(line))
     if world > 1:

@@ -224,6 +224,37 @@ brisk_status brisk_last_device_status(void *workspace, int32_t clear, void *stre
 /* Human-readable name of a status code (static storage). */
 const char *brisk_status_string(brisk_status status);
 
+/* ---- Acceptance profile and risk-reward position weights (Sec. 2.2; Sec. 3.2 Eqs. 2-3) ----
+ *
+ * The paper estimates the per-position acceptance a_i of a verified block as one minus the
+ * rejection rate at position i among the blocks whose verification reached i, and turns the
+ * profile into tokens per forward (TPF) and position weights for the proposal loss. */
+
+/* Adds one block step's accepted lengths to running counts (device): for every position
+ * i < L, counts[i] += #{b : accepted_len[b] >= i} (blocks that reached i) and
+ * counts[L + i] += #{b : accepted_len[b] >= i + 1} (blocks that accepted i). accepted_len
+ * [B] int32 (device, values in 0..L, the output of brisk_verify_block / brisk_decode_tail);
+ * counts [2L] uint64 (device, caller-owned, zeroed by the caller before the first step).
+ * Integer sums: the counts do not depend on timing. Lengths outside 0..L are clamped.
+ * 1 <= L <= 64, B >= 0. */
+brisk_status brisk_acceptance_counts(const int32_t *accepted_len, int32_t B, int32_t L,
+                                     unsigned long long *counts, void *stream);
+
+/* Host-side (no device work). For a profile a[0..M-1] (a_i in [0, 1], position i of the block)
+ * and per-length committed tokens g[0..M] and forward costs c[0..M] (Eq. 2), writes
+ * tpf = sum_k Pr(L=k) g_k / sum_k Pr(L=k) c_k with Pr(L=k) = A_k (1 - a_k) for k < M and A_M
+ * for k = M (A_k = a_0 ... a_{k-1}); w_raw[i] = -dFPT/dz_i with FPT = 1/TPF and
+ * z_i = log(a_i / (1 - a_i)); w_bar[i] = M w_raw[i] / (sum_j w_raw[j] + eps) (Eq. 3). g or c
+ * NULL means g_k = k + 1 and c_k = 1 (one guaranteed token, unit cost: TPF = 1 + sum A_k).
+ * Any output pointer may be NULL. 1 <= M <= 64; BRISK_ERR_INVALID_ARG for a NULL profile, an
+ * a_i outside [0, 1] or a zero expected cost. */
+brisk_status brisk_acceptance_weights(int32_t M, const double *a, const double *g, const double *c,
+                                      double eps, double *tpf, double *w_raw, double *w_bar);
+
+/* Host-side: tokens per forward of the ISD stride-N rule at constant rejection r (Sec. 2.2):
+ * (2 + sum_{i=1}^{N-2} (1-r)^i) / (2 - (1-r)^{N-1}); NaN for N < 2 or r outside [0, 1]. */
+double brisk_tpf_isd(int32_t N, double r);
+
 #ifdef __cplusplus
 }
 #endif

@@ -76,6 +76,10 @@ _SIGS = [
     ("brisk_kernels_per_tail", ctypes.c_int32, [ctypes.POINTER(Dims)]),
     ("brisk_last_device_status", ctypes.c_int, [_vp, ctypes.c_int32, _vp]),
     ("brisk_status_string", ctypes.c_char_p, [ctypes.c_int]),
+    ("brisk_acceptance_counts", ctypes.c_int, [_vp, ctypes.c_int32, ctypes.c_int32, _vp, _vp]),
+    ("brisk_acceptance_weights", ctypes.c_int,
+     [ctypes.c_int32, _vp, _vp, _vp, ctypes.c_double, _vp, _vp, _vp]),
+    ("brisk_tpf_isd", ctypes.c_double, [ctypes.c_int32, ctypes.c_double]),
 ]
 
 
@@ -254,3 +258,36 @@ class DecodeTail:
 def mode_ids(select_mode: str, verify_mode: str):
     return (SELECT_SAMPLE if select_mode == "sample" else SELECT_GREEDY,
             VERIFY_STOCHASTIC if verify_mode == "stochastic" else VERIFY_GREEDY)
+
+
+# ---------------------------------------------------------------- acceptance profile
+
+def acceptance_counts(accepted_len: torch.Tensor, L: int, counts: torch.Tensor, stream=None) -> None:
+    """Adds one step's accepted lengths ([B] int32, device) to running per-position counts
+    (counts: [2L] int64 device tensor used as uint64; reached first, then accepted)."""
+    if accepted_len.dtype != torch.int32 or counts.dtype != torch.int64 or counts.numel() != 2 * L:
+        raise ValueError("accepted_len int32 [B], counts int64 [2L]")
+    _check(lib().brisk_acceptance_counts(_p(accepted_len), int(accepted_len.numel()), int(L),
+                                         _p(counts), _stream(stream)), "acceptance_counts")
+
+
+def acceptance_weights(a, g=None, c=None, eps: float = 1e-8):
+    """TPF, w_raw and the mean-one w_bar of a profile a[0..M-1] (host, float64)."""
+    import numpy as np
+    a = np.ascontiguousarray(a, dtype=np.float64)
+    M = a.size
+    gg = None if g is None else np.ascontiguousarray(g, dtype=np.float64)
+    cc = None if c is None else np.ascontiguousarray(c, dtype=np.float64)
+    if (gg is not None and gg.size != M + 1) or (cc is not None and cc.size != M + 1):
+        raise ValueError("g and c need M + 1 entries")
+    tpf = ctypes.c_double()
+    w_raw = np.empty(M)
+    w_bar = np.empty(M)
+    vp = lambda x: None if x is None else x.ctypes.data_as(ctypes.c_void_p)
+    _check(lib().brisk_acceptance_weights(M, vp(a), vp(gg), vp(cc), float(eps), ctypes.byref(tpf),
+                                          vp(w_raw), vp(w_bar)), "acceptance_weights")
+    return tpf.value, w_raw, w_bar
+
+
+def tpf_isd(N: int, r: float) -> float:
+    return float(lib().brisk_tpf_isd(int(N), float(r)))
