@@ -6,12 +6,12 @@
  * Generation for Diffusion Language Models", Sec. 3.3 and Algorithm 1(b)):
  *
  *   1. candidates: log-sum-exp over the full vocabulary and the ordered Top-K
- *      of every masked position (Sec. 3.3 "C_i = TopK(q_i, K)"; App. C.2);
+ *      of every masked position (Sec. 3.3 "C_i = TopK(q_i, K)"; App. C.3);
  *   2. the prefix-conditioned corrector, which reranks only those K
  *      candidates with a minimal-GRU state that reads the tokens selected
- *      earlier in the block (Sec. 3.3 Eqs. 4-5; App. C.2 Eq. 7);
+ *      earlier in the block (Sec. 3.3 Eqs. 4-5; App. C.3 Eq. 9);
  *   3. left-to-right verification against the verifier distribution up to the
- *      first rejection (Sec. 3.1; Sec. 3.3; App. B Eq. 8).
+ *      first rejection (Sec. 3.1; Sec. 3.3; App. B Eq. 6).
  *
  * Conventions shared by every entry point:
  *  - Every tensor argument is caller-owned device memory, row-major and dense
@@ -65,7 +65,7 @@ typedef enum brisk_verify_mode { BRISK_VERIFY_GREEDY = 0, BRISK_VERIFY_STOCHASTI
 
 /* Problem sizes. B sequences, block length L (the paper's M), vocabulary V, backbone width d,
  * K candidates, corrector width r. The corrector state has S = 2r dimensions; the position
- * embedding and the feature projection have 16 (App. C.2 head configuration, with
+ * embedding and the feature projection have 16 (App. C.3 head configuration, with
  * rank = hidden projection = token projection = r).
  * Limits: B >= 1; 1 <= L <= 64; 4 <= K <= 32; V >= K; d >= 8 and d % 8 == 0;
  * 16 <= r <= 512 and r % 16 == 0. */
@@ -75,7 +75,7 @@ typedef struct brisk_dims {
   int32_t hidden_dtype;   /* brisk_dtype of hidden, h_ctx, every weight and E_in/E_out */
 } brisk_dims;
 
-/* Corrector parameters psi and the frozen vocabulary rows (App. C.2), device pointers in
+/* Corrector parameters psi and the frozen vocabulary rows (App. C.3), device pointers in
  * hidden_dtype, row-major:
  *   E_in  [V, d]   frozen input token embedding E
  *   E_out [V, d]   frozen LM-head rows E_out
@@ -133,14 +133,14 @@ size_t brisk_workspace_bytes(const brisk_dims *dims);
 size_t brisk_tables_bytes(const brisk_dims *dims);
 
 /* Fold the frozen vocabulary rows into the corrector's weights, once per weight set
- * (App. C.2: E_in, E_out and the backbone stay frozen, so P_e E_in(v), W_c E_out(v) and
+ * (App. C.3: E_in, E_out and the backbone stay frozen, so P_e E_in(v), W_c E_out(v) and
  * their products with the GRU and residual matrices are fixed per token). Fills `tables`
  * (brisk_tables_bytes(dims) bytes). Must run before brisk_corrector_select /
  * brisk_decode_tail with these params; `params` buffers may be freed afterwards. */
 brisk_status brisk_corrector_prepare(const brisk_dims *dims, const brisk_params *params,
                                      void *tables, void *stream);
 
-/* Step 1 (Sec. 3.3 "C_i = TopK(q_i, K)"; App. C.2 ordered candidate set S_j): for every row
+/* Step 1 (Sec. 3.3 "C_i = TopK(q_i, K)"; App. C.3 ordered candidate set S_j): for every row
  * (b, i) of logits_q [B, L, V]: lse_q = max + log sum exp(l - max) over all V, the K ids of
  * largest logit ordered by (logit descending, id ascending) in cand_ids [B, L, K], and
  * cand_logprob = l(id) - lse_q. */
@@ -167,7 +167,7 @@ brisk_status brisk_topk_candidates_noalloc(const brisk_dims *dims, const void *l
                                            int32_t *cand_ids, float *cand_logprob, float *lse_q,
                                            void *stream);
 
-/* Step 2 (Sec. 3.3 Eqs. 4-5; App. C.2 Eq. 7; Algorithm 1(b) loop): per sequence, sequentially
+/* Step 2 (Sec. 3.3 Eqs. 4-5; App. C.3 Eq. 9; Algorithm 1(b) loop): per sequence, sequentially
  * over positions, the minimal-GRU corrector state, the gated low-rank residual on the K
  * candidates and Select. Reads the step-1 outputs (cand_ids, cand_logprob) and logits_q
  * (for the confidence features), hidden [B, L, d], h_ctx [B, d], x0 [B]; u_sel [B, L] is
@@ -181,7 +181,7 @@ brisk_status brisk_corrector_select(const brisk_dims *dims, const brisk_params *
                                     int32_t *sel_tokens, float *refined,
                                     void *workspace, void *stream);
 
-/* Step 3 (Sec. 3.1 accept-prefix; Sec. 3.3 speculative sampling; App. B Eq. 8 strict u < alpha):
+/* Step 3 (Sec. 3.1 accept-prefix; Sec. 3.3 speculative sampling; App. B Eq. 6 strict u < alpha):
  * verifier row statistics over logits_p [B, L, V], then per sequence left to right to the first
  * rejection. Greedy: accept iff sel_tokens[b,i] is the verifier argmax (lowest id on ties); the
  * correction is that argmax. Stochastic: pi_i is softmax(refined) on cand_ids for sample Select and

@@ -10,11 +10,11 @@ What it follows (section / equation of the paper, "From Position Risks to
 Block Survival: Faster Generation for Diffusion Language Models"):
 
 1. Candidates (Sec. 3.3, "C_i = TopK(q_i, K)" on the normalised proposal
-   q_i; App. C.2, the ordered candidate set S_j that the head never expands):
+   q_i; App. C.3, the ordered candidate set S_j that the head never expands):
    log-partition LSE = m + log sum exp(l - m); the K ids of largest logit,
    ordered by (logit descending, id ascending); cand_logprob = l - LSE.
 2. Corrector (Sec. 3.3, Eq. 4 recurrent state and Eq. 5 candidate residual;
-   App. C.2 head details and Eq. 7 residual logits; Algorithm 1(b)):
+   App. C.3 head details and Eq. 9 residual logits; Algorithm 1(b)):
    u_0 = Init(h_c, E(x_0)); per position i the minimal GRU reads the
    concatenation [P_h m_i ; P_e E_in(x_{i-1}) ; pos_i ; P_phi phi_i],
    d_{i,k} = <W_s s_i, W_c E_out(c_{i,k})>,
@@ -22,7 +22,7 @@ Block Survival: Faster Generation for Diffusion Language Models"):
    refined_{i,k} = log q_i(c_{i,k}) + gamma_i d_{i,k}, then Select.
 3. Verification (Sec. 3.1, accept-prefix semantics; Sec. 3.3, standard
    speculative sampling with acceptance min{1, p/pi} and resampling from the
-   normalised [p - pi]_+; App. B, Eq. 8, strict u < alpha): left to right up
+   normalised [p - pi]_+; App. B, Eq. 6, strict u < alpha): left to right up
    to the first rejection.
 
 Readings taken where the paper is silent or ambiguous (each is listed in the
@@ -62,7 +62,7 @@ class OracleError(ValueError):
 
 
 # ---------------------------------------------------------------------------
-# Step 1: log-partition and Top-K (Sec. 3.3, App. C.2)
+# Step 1: log-partition and Top-K (Sec. 3.3, App. C.3)
 # ---------------------------------------------------------------------------
 
 def log_partition(row: np.ndarray) -> float:
@@ -96,7 +96,7 @@ def verifier_argmax(row: np.ndarray) -> int:
 
 
 # ---------------------------------------------------------------------------
-# Step 2: the prefix-conditioned corrector (Sec. 3.3 Eqs. 4-5, App. C.2 Eq. 7)
+# Step 2: the prefix-conditioned corrector (Sec. 3.3 Eqs. 4-5, App. C.3 Eq. 9)
 # ---------------------------------------------------------------------------
 
 def sigmoid(x):
@@ -104,7 +104,7 @@ def sigmoid(x):
 
 
 def confidence_features(row: np.ndarray, top4: Sequence[int], prev: int) -> np.ndarray:
-    """phi_i (App. C.2): top1-top2 gap, top1-top4 gap, [prev = top1], [prev in top4],
+    """phi_i (App. C.3): top1-top2 gap, top1-top4 gap, [prev = top1], [prev in top4],
     top1 minus the logit of the previous token, all on position i's own proposal row."""
     t1, t2, t4 = int(top4[0]), int(top4[1]), int(top4[3])
     return np.array([
@@ -156,7 +156,7 @@ def init_state(p: Params, h_c: np.ndarray, x0: int) -> np.ndarray:
 
 
 def proposal_law(refined: np.ndarray, mode: str, sel_rank: int) -> np.ndarray:
-    """pi_i over the K candidates induced by the selection rule (App. C.2): softmax of
+    """pi_i over the K candidates induced by the selection rule (App. C.3): softmax of
     the refined scores for sampling; greedy selection puts all mass on the selected rank."""
     if mode == SAMPLE:
         m = np.max(refined)
@@ -245,7 +245,7 @@ def corrector_sequence(p: Params, hidden: np.ndarray, h_c: np.ndarray, x0: int,
 
 
 # ---------------------------------------------------------------------------
-# Step 3: verification through the first rejection (Sec. 3.1, 3.3; App. B Eq. 8)
+# Step 3: verification through the first rejection (Sec. 3.1, 3.3; App. B Eq. 6)
 # ---------------------------------------------------------------------------
 
 @dataclass

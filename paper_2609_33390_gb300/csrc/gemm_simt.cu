@@ -1,6 +1,6 @@
 // Plain tiled fp32 dense products and a conversion copy. They serve the one-off
 // folding of the frozen vocabulary rows into the corrector tables
-// (App. C.2: E, E_out and the backbone are frozen at inference) and the fp32
+// (App. C.3: E, E_out and the backbone are frozen at inference) and the fp32
 // configurations; every product accumulates in fp32.
 #include "brisk_internal.cuh"
 

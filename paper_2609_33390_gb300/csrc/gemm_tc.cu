@@ -11,7 +11,7 @@
 // drains what it started and frees its TMEM.
 //
 // Used for the corrector's one dense contraction (the MASK hidden states times
-// the hidden projection, App. C.2 "64-dimensional projection of the MASK
+// the hidden projection, App. C.3 "64-dimensional projection of the MASK
 // hidden state") and for the products that follow it, where an fp32 operand
 // enters as the sum of three bf16 parts (hi + mid + lo) so that bf16 tensor
 // cores keep fp32-level accuracy.

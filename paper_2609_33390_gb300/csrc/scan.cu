@@ -1,6 +1,6 @@
 // Corrector scan and verification, one CTA per sequence.
 //
-// Corrector (Sec. 3.3 Eqs. 4-5; App. C.2 Eq. 7; Algorithm 1(b) loop). The
+// Corrector (Sec. 3.3 Eqs. 4-5; App. C.3 Eq. 9; Algorithm 1(b) loop). The
 // minimal-GRU pre-activations are linear in the input blocks
 // [P_h m_i ; P_e E_in(x_{i-1}) ; pos_i ; P_phi phi_i], so each block's share is
 // read from a precomputed source:
@@ -13,7 +13,7 @@
 // sequential per position is O(S) element work, K+1 dot products of length S
 // and the K-way Select.
 //
-// Verification (Sec. 3.1; Sec. 3.3; App. B Eq. 8) runs in the same CTA after
+// Verification (Sec. 3.1; Sec. 3.3; App. B Eq. 6) runs in the same CTA after
 // the scan, or alone (brisk_verify_block), through the same device code.
 #include "brisk_internal.cuh"
 
@@ -344,7 +344,7 @@ __device__ void verify_sequence(const ScanArgs& a, const Smem& sm, int b) {
     a.out_tokens[(size_t)b * L + t] = t < j ? sm.sel[t] : (t == j ? corr : -1);
 }
 
-// Verification of one sequence per CTA (Sec. 3.1; Sec. 3.3; App. B Eq. 8), reading the
+// Verification of one sequence per CTA (Sec. 3.1; Sec. 3.3; App. B Eq. 6), reading the
 // selections and refined scores the corrector wrote.
 __global__ void __launch_bounds__(SCAN_THREADS)
 verify_kernel(const __grid_constant__ ScanArgs a) {
@@ -473,7 +473,7 @@ __device__ __forceinline__ void gather_logits(const void* logits, int dt, int n,
   }
 }
 
-// The sequential corrector (Sec. 3.3 Eqs. 4-5; App. C.2 Eq. 7; Algorithm 1(b) loop), one CTA of
+// The sequential corrector (Sec. 3.3 Eqs. 4-5; App. C.3 Eq. 9; Algorithm 1(b) loop), one CTA of
 // NW warps per sequence. Lane l of warp w owns the 4-element state chunks
 // c = l + 32 (w + NW m), m < CMC. The residual dots and the gate are reduced with warp
 // shuffles, then across the warps through shared memory (one block barrier a position), and
@@ -610,7 +610,7 @@ corrector_kernel(const __grid_constant__ ScanArgs a) {
         tnh[m] = ldcg4(Tn + S + 4 * cc[m]);
       }
     }
-    // confidence features of position i (App. C.2)
+    // confidence features of position i (App. C.3)
     const float l0 = sm.top[i * 3 + 0];
     float phi[5];
     phi[0] = l0 - sm.top[i * 3 + 1];

@@ -1,5 +1,5 @@
 // Vocabulary sweep: per logit row, the log-partition and the ordered top-K
-// (Sec. 3.3 "C_i = TopK(q_i, K)"; App. C.2 ordered candidate set), and for
+// (Sec. 3.3 "C_i = TopK(q_i, K)"; App. C.3 ordered candidate set), and for
 // verifier rows the argmax (lowest id on ties) and the log-partition.
 //
 // Work unit: one warp sweeps one chunk of one row with coalesced 16-byte

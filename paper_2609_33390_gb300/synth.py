@@ -248,7 +248,7 @@ WORKLOADS = {
 def weight_shapes(wl: Workload) -> dict:
     """Corrector parameter shapes (row-major) under the width mapping
     rank = hidden projection = token projection = r, state S = 2r, position and
-    feature projections 16 (App. C.2, head configuration table)."""
+    feature projections 16 (App. C.3, head configuration table)."""
     r, S, d = wl.r, wl.S, wl.d
     return {
         "P_h": (r, d), "P_e": (r, d), "P_phi": (16, 5), "pos": (wl.L, 16),

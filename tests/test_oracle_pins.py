@@ -91,7 +91,7 @@ def test_verifier_argmax_lowest_id_on_ties():
 
 
 # ---------------------------------------------------------------------------
-# Confidence features: a worked example from the definitions in App. C.2
+# Confidence features: a worked example from the definitions in App. C.3
 # ---------------------------------------------------------------------------
 
 def test_features_worked_example():
