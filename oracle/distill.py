@@ -41,8 +41,9 @@ def _log_softmax(x):
 
 
 def reached_mask(accepted_len, L: int):
-    """m[b, j] = 1 for j <= min(accepted_len[b], L - 1)."""
-    a = np.asarray(accepted_len, dtype=np.int64)
+    """m[b, j] = 1 for j <= min(accepted_len[b], L - 1); lengths outside 0..L are clamped
+    (an accepted length is at least 0, so position 0 is always reached)."""
+    a = np.clip(np.asarray(accepted_len, dtype=np.int64), 0, L)
     j = np.arange(L)
     return (j[None, :] <= np.minimum(a, L - 1)[:, None]).astype(np.float64)
 
