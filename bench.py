@@ -342,6 +342,20 @@ def run_ours(args):
     reach_h, accept_h = counts_h[:wl.L], counts_h[wl.L:]
     prof_a = [accept_h[i] / reach_h[i] if reach_h[i] else 0.0 for i in range(wl.L)]
     prof_tpf, _, prof_w = brisk.acceptance_weights(prof_a)
+    # distillation loss of the head (App. C.3) on one block's outputs: kernel time, untimed above
+    full = tail.alloc_outputs(full=True)
+    tail.tail(pool[0], sm, vm, out=full)
+    dl_args = (pool[0]["logits_p"], full["cand_ids"], full["cand_logprob"], full["refined"],
+               full["accepted_len"])
+    for _ in range(3):
+        tail.distill_loss(*dl_args)
+    d0, d1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    d0.record(stream)
+    for _ in range(20):
+        tail.distill_loss(*dl_args)
+    d1.record(stream)
+    torch.cuda.synchronize()
+    distill_us = 1000.0 * d0.elapsed_time(d1) / 20
     sweep_q_ms = [events[s][0].elapsed_time(events[s][1]) for s in range(args.warmup, nsteps)]
     sweep_p_ms = [events[s][2].elapsed_time(events[s][3]) for s in range(args.warmup, nsteps)]
     sweep_ms = [q + p for q, p in zip(sweep_q_ms, sweep_p_ms)]
@@ -412,6 +426,7 @@ def run_ours(args):
                                "positions_shown": min(8, wl.L),
                                "tpf_unit_cost": prof_tpf,
                                "w_bar": [round(x, 4) for x in prof_w[:8]]},
+        "distill_loss_us": distill_us,
     }
     print(json.dumps(line))
     if world > 1:

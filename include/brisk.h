@@ -251,6 +251,24 @@ brisk_status brisk_acceptance_counts(const int32_t *accepted_len, int32_t B, int
 brisk_status brisk_acceptance_weights(int32_t M, const double *a, const double *g, const double *c,
                                       double eps, double *tpf, double *w_raw, double *w_bar);
 
+/* ---- Distillation loss of the refinement head (App. C.3, Eq. 10) ----
+ *
+ * The training objective of the corrector on a batch of blocks: at every reached position j
+ * (j <= min(accepted_len[b], L-1): the accepted prefix and the first rejected position),
+ * CE(p_S, r) + beta KL(q_S || r), where p_S = the verifier distribution restricted to the K
+ * candidates of position j and renormalised (from logits_p at cand_ids), q_S = the proposal
+ * distribution restricted to them (from cand_logprob), r = softmax(refined); the loss is one
+ * mean over all reached positions of the batch (the paper uses beta = 0.01).
+ * logits_p [B, L, V] (dims.logits_dtype), cand_ids / cand_logprob / refined [B, L, K],
+ * accepted_len [B] int32 (values outside 0..L are clamped), all device. Writes loss [1] f32
+ * (device) and, unless grad_refined is NULL, d loss / d refined [B, L, K] f32 (device; zero at
+ * unreached positions). The loss does not depend on timing. An out-of-range candidate id is
+ * replaced by 0 and reported as BRISK_ERR_INVALID_ARG in the device status. */
+brisk_status brisk_distill_loss(const brisk_dims *dims, const void *logits_p,
+                                const int32_t *cand_ids, const float *cand_logprob,
+                                const float *refined, const int32_t *accepted_len, float beta,
+                                float *loss, float *grad_refined, void *workspace, void *stream);
+
 /* Host-side: tokens per forward of the ISD stride-N rule at constant rejection r (Sec. 2.2):
  * (2 + sum_{i=1}^{N-2} (1-r)^i) / (2 - (1-r)^{N-1}); NaN for N < 2 or r outside [0, 1]. */
 double brisk_tpf_isd(int32_t N, double r);

@@ -80,6 +80,8 @@ _SIGS = [
     ("brisk_acceptance_weights", ctypes.c_int,
      [ctypes.c_int32, _vp, _vp, _vp, ctypes.c_double, _vp, _vp, _vp]),
     ("brisk_tpf_isd", ctypes.c_double, [ctypes.c_int32, ctypes.c_double]),
+    ("brisk_distill_loss", ctypes.c_int,
+     [ctypes.POINTER(Dims), _vp, _vp, _vp, _vp, _vp, ctypes.c_float, _vp, _vp, _vp, _vp]),
 ]
 
 
@@ -221,6 +223,18 @@ class DecodeTail:
             int(select_mode), int(verify_mode), _p(u_acc), _p(u_res), _p(a), _p(out), _p(corr),
             _p(self.workspace), _stream(stream)), "verify")
         return {"accepted_len": a, "out_tokens": out, "correction": corr}
+
+    def distill_loss(self, logits_p, cand_ids, cand_logprob, refined, accepted_len, beta=0.01,
+                     with_grad=True, stream=None):
+        """Distillation loss of the refinement head (App. C.3, Eq. 10) and its gradient in the
+        refined scores."""
+        loss = self._f32(1)
+        grad = self._f32(self.B, self.L, self.K) if with_grad else None
+        _check(lib().brisk_distill_loss(
+            ctypes.byref(self.dims), _p(logits_p), _p(cand_ids), _p(cand_logprob), _p(refined),
+            _p(accepted_len), float(beta), _p(loss), _p(grad), _p(self.workspace),
+            _stream(stream)), "distill_loss")
+        return {"loss": loss, "grad": grad}
 
     def alloc_outputs(self, full=True):
         B, L, K = self.B, self.L, self.K

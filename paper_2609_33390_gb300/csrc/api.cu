@@ -29,7 +29,7 @@ inline size_t esize(int dt) { return dt == BRISK_DT_BF16 ? 2 : 4; }
 // ---------------------------------------------------------------- workspace layout
 struct WsLayout {
   size_t status, counters, part_val, part_id, part_m, part_s, argmax_p, lse_p;
-  size_t cand_ids, cand_logprob, lse_q, sel, refined, Hm, G, G0, total;
+  size_t cand_ids, cand_logprob, lse_q, sel, refined, Hm, G, G0, distill, total;
   int nchunk_q, nchunk_p, KP;   // chunks per proposal row (row layout) and verifier row (split)
 };
 
@@ -59,6 +59,7 @@ WsLayout ws_layout(const brisk_dims* d) {
   w.Hm = take(6 * (BL + d->B) * d->r);   // fp32 [BL+B, r] or bf16 [BL+B, 3r]
   w.G = take(sizeof(float) * BL * 2 * S);
   w.G0 = take(sizeof(float) * d->B * S);
+  w.distill = take(sizeof(float) * d->B);   // per-sequence loss partials of brisk_distill_loss
   w.total = o;
   return w;
 }
@@ -543,6 +544,36 @@ brisk_status brisk_last_device_status(void* ws, int32_t clear, void* stream) {
     BRISK_CUDA(cudaStreamSynchronize(st));
   }
   return static_cast<brisk_status>(h);
+}
+
+
+brisk_status brisk_distill_loss(const brisk_dims* d, const void* logits_p, const int32_t* cand_ids,
+                                const float* cand_logprob, const float* refined,
+                                const int32_t* accepted_len, float beta, float* loss,
+                                float* grad_refined, void* ws, void* stream) {
+  if (!dims_ok(d) || !logits_p || !cand_ids || !cand_logprob || !refined || !accepted_len ||
+      !loss || !ws || !aligned(ws, ALIGN) || !aligned(logits_p, esize(d->logits_dtype)) ||
+      !(beta >= 0.f))
+    return BRISK_ERR_INVALID_ARG;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const WsLayout w = ws_layout(d);
+  brisk_status s = clear_ws(w, d, ws, st);
+  if (s != BRISK_OK) return s;
+  DistillArgs a{};
+  a.B = d->B; a.L = d->L; a.V = d->V; a.K = d->K; a.logits_dt = d->logits_dtype;
+  a.logits_p = logits_p;
+  a.cand_ids = cand_ids;
+  a.cand_logprob = cand_logprob;
+  a.refined = refined;
+  a.accepted_len = accepted_len;
+  a.beta = beta;
+  a.loss = loss;
+  a.grad = grad_refined;
+  a.partial = at<float>(ws, w.distill);
+  a.arrivals = at<int32_t>(ws, w.status) + 16;   // a word of the (cleared) status block
+  a.status = at<int32_t>(ws, w.status);
+  BRISK_CUDA(launch_distill(a, st));
+  return BRISK_OK;
 }
 
 }  // extern "C"

@@ -280,6 +280,23 @@ struct ScanArgs {
   int32_t* status;
 };
 
+// ---------------------------------------------------------------- distillation loss
+struct DistillArgs {
+  int B, L, V, K, logits_dt;
+  const void* logits_p;        // [B, L, V] verifier logits
+  const int32_t* cand_ids;     // [B, L, K]
+  const float* cand_logprob;   // [B, L, K]
+  const float* refined;        // [B, L, K]
+  const int32_t* accepted_len; // [B]
+  float beta;
+  float* loss;                 // [1]
+  float* grad;                 // [B, L, K] or nullptr
+  float* partial;              // [B] per-sequence loss sums (workspace)
+  int32_t* arrivals;           // zero on entry (workspace)
+  int32_t* status;
+};
+cudaError_t launch_distill(const DistillArgs& a, cudaStream_t stream);
+
 size_t scan_smem_bytes(int L, int K, int S, int V);
 cudaError_t launch_scan(const ScanArgs& a, cudaStream_t stream);
 
