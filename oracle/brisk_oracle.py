@@ -201,13 +201,17 @@ def corrector_sequence(p: Params, hidden: np.ndarray, h_c: np.ndarray, x0: int,
                        rows_q: Callable[[int], np.ndarray], cand_ids: np.ndarray,
                        cand_logprob: np.ndarray, top4: np.ndarray, mode: str = GREEDY,
                        u_sel: Optional[np.ndarray] = None,
-                       force: Optional[Dict[int, int]] = None) -> CorrectorTrace:
+                       force: Optional[Dict[int, int]] = None,
+                       prefix_ranks: Optional[np.ndarray] = None) -> CorrectorTrace:
     """Algorithm 1(b) lines for i = 1..M of one sequence (0-based i here).
 
     hidden: [L, d] MASK hidden states m_i; h_c: [d]; x0: anchor token;
     rows_q(i): proposal logit row i; cand_ids/cand_logprob: [L, K] from step 1;
     top4: [L, 4] the row's four highest ids (for phi); force: {i: rank} overrides
-    Select at position i (used where two choices are equally correct).
+    Select at position i (used where two choices are equally correct);
+    prefix_ranks: [L] candidate ranks of a fixed prefix; when given, the token before
+    position i + 1 is cand_ids[i][prefix_ranks[i]] instead of the selection at i (the
+    same-state replay of App. B conditions the head on the factual base prefix).
     """
     L, K = cand_ids.shape
     s = init_state(p, h_c, x0)                          # s_{-1} = u_0
@@ -240,8 +244,62 @@ def corrector_sequence(p: Params, hidden: np.ndarray, h_c: np.ndarray, x0: int,
         out.gamma[i] = gamma
         out.features[i] = phi
         out.margin[i] = margin
-        prev = int(cand_ids[i][k])
+        prev = int(cand_ids[i][k if prefix_ranks is None else int(prefix_ranks[i])])
     return out
+
+
+# ---------------------------------------------------------------------------
+# Same-state replay diagnostics (App. B, "Same-state replay", Eq. 6)
+# ---------------------------------------------------------------------------
+
+def base_ranks(cand_logprob: np.ndarray, mode: str = GREEDY,
+               u_sel: Optional[np.ndarray] = None) -> np.ndarray:
+    """The head-off (factual base) selection: the Select rule applied to the base scores
+    log q (rank 0 under greedy; the inverse-CDF draw from the base law under sampling)."""
+    L = cand_logprob.shape[0]
+    if mode == SAMPLE:
+        return np.array([sample_pick(cand_logprob[i], float(u_sel[i]))[0] for i in range(L)])
+    return np.array([greedy_pick(cand_logprob[i]) for i in range(L)])
+
+
+@dataclass
+class ReplayResult:
+    base_rank: np.ndarray       # [L]
+    head_rank: np.ndarray       # [L] the head's selection on the factual base prefix
+    alpha_base: np.ndarray      # [L] min(1, p/q) at the base token
+    alpha_head: np.ndarray      # [L]
+    first_breaker: int          # first position whose base token the draw rejects (L if none)
+    intervention: np.ndarray    # [L] bool: head token != base token
+    rescue: np.ndarray          # [L] bool: at the first breaker, the draw accepts the head token
+    regression: np.ndarray      # [L] bool: before the first breaker, the draw rejects the head
+    trace: CorrectorTrace
+
+
+def replay_sequence(p: Params, rows_q, rows_p, hidden, h_c, x0, cand_ids, cand_logprob, top4,
+                    u_acc, mode: str = GREEDY, u_sel=None) -> ReplayResult:
+    """Same-state replay: with the factual base prefix, the base q_i (normalised over the full
+    vocabulary), the verifier p_i and the draw u_i fixed, only the token at each position
+    changes: alpha_i(x) = min(1, p_i(x) / q_i(x)), J_i(x) = [u_i < alpha_i(x)] (App. B, Eq. 6).
+    A rescue is J(x_base) = 0 and J(x_head) = 1 at the factual first breaker; a regression is
+    J(x_base) = 1 and J(x_head) = 0 at a factual accepted position (one before the breaker)."""
+    L, K = cand_ids.shape
+    b = base_ranks(cand_logprob, mode, u_sel)
+    tr = corrector_sequence(p, hidden, h_c, int(x0), rows_q, cand_ids, cand_logprob, top4, mode,
+                            u_sel, prefix_ranks=b)
+    h = tr.sel_rank.copy()
+
+    def alpha(i, k):
+        row = np.asarray(rows_p(i), dtype=np.float64)
+        lp = float(row[int(cand_ids[i][k])]) - log_partition(row)
+        return min(1.0, float(np.exp(lp - cand_logprob[i][k])))
+
+    ab = np.array([alpha(i, b[i]) for i in range(L)])
+    ah = np.array([alpha(i, h[i]) for i in range(L)])
+    jb = np.asarray(u_acc, dtype=np.float64) < ab
+    jh = np.asarray(u_acc, dtype=np.float64) < ah
+    fb = next((i for i in range(L) if not jb[i]), L)
+    pos = np.arange(L)
+    return ReplayResult(b, h, ab, ah, fb, h != b, (pos == fb) & jh, (pos < fb) & ~jh, tr)
 
 
 # ---------------------------------------------------------------------------
