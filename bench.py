@@ -356,6 +356,21 @@ def run_ours(args):
     d1.record(stream)
     torch.cuda.synchronize()
     distill_us = 1000.0 * d0.elapsed_time(d1) / 20
+    # same-state replay diagnostics (App. B) over the block pool: rates and the call's time
+    n_fb = n_res = n_int = n_acc = n_reg = 0
+    for blk in pool:
+        fl = tail.replay(blk, sm)["flags"]
+        n_fb += int(((fl & 4) != 0).sum())
+        n_int += int(((fl & 4) != 0).logical_and((fl & 8) != 0).sum())
+        n_res += int(((fl & 16) != 0).sum())
+        n_acc += int(((fl & 1) != 0).logical_and((fl & 4) == 0).sum())
+        n_reg += int(((fl & 32) != 0).sum())
+    d0.record(stream)
+    for _ in range(5):
+        tail.replay(pool[0], sm)
+    d1.record(stream)
+    torch.cuda.synchronize()
+    replay_us = 1000.0 * d0.elapsed_time(d1) / 5
     sweep_q_ms = [events[s][0].elapsed_time(events[s][1]) for s in range(args.warmup, nsteps)]
     sweep_p_ms = [events[s][2].elapsed_time(events[s][3]) for s in range(args.warmup, nsteps)]
     sweep_ms = [q + p for q, p in zip(sweep_q_ms, sweep_p_ms)]
@@ -427,6 +442,11 @@ def run_ours(args):
                                "tpf_unit_cost": prof_tpf,
                                "w_bar": [round(x, 4) for x in prof_w[:8]]},
         "distill_loss_us": distill_us,
+        "replay": {"first_breakers": n_fb,
+                   "intervention_rate_at_breakers": n_int / max(1, n_fb),
+                   "rescue_rate_at_breakers": n_res / max(1, n_fb),
+                   "regression_rate_at_accepted": n_reg / max(1, n_acc),
+                   "call_us": replay_us},
     }
     print(json.dumps(line))
     if world > 1:

@@ -251,6 +251,30 @@ brisk_status brisk_acceptance_counts(const int32_t *accepted_len, int32_t B, int
 brisk_status brisk_acceptance_weights(int32_t M, const double *a, const double *g, const double *c,
                                       double eps, double *tpf, double *w_raw, double *w_bar);
 
+/* ---- Same-state replay diagnostics (App. B, "Same-state replay", Eq. 6) ----
+ *
+ * Runs the candidates, the verifier rows' log-partition and the corrector with the head
+ * conditioned on the factual base prefix (the token fed forward at every position is the base
+ * selection: the Select rule applied to the base scores log q with the same draw u_sel, i.e.
+ * rank 0 under greedy selection), then scores the base token and the head's token of every
+ * position under one shared draw: alpha_i(x) = min(1, p_i(x) / q_i(x)) with q_i the proposal
+ * normalised over the full vocabulary and p_i the verifier, J_i(x) = [u_acc_i < alpha_i(x)].
+ * Inputs as brisk_corrector_select plus logits_p [B, L, V] and u_acc [B, L] f32 (device).
+ * Outputs (device): head_tokens [B, L] int32; flags [B, L] int32 with bit 0 = J(base),
+ * bit 1 = J(head), bit 2 = first breaker (the first position whose base token the draw
+ * rejects), bit 3 = intervention (head token != base token), bit 4 = rescue (J(base) = 0 and
+ * J(head) = 1 at the first breaker), bit 5 = regression (J(head) = 0 at a position before the
+ * first breaker, where J(base) = 1); first_breaker [B] int32 (L if none); refined [B, L, K]
+ * f32 or NULL. */
+brisk_status brisk_replay_diagnostics(const brisk_dims *dims, const brisk_params *params,
+                                      const void *tables, const void *hidden, const void *h_ctx,
+                                      const int32_t *x0, const void *logits_q,
+                                      const void *logits_p, int32_t select_mode,
+                                      const float *u_sel, const float *u_acc,
+                                      int32_t *head_tokens, int32_t *flags,
+                                      int32_t *first_breaker, float *refined, void *workspace,
+                                      void *stream);
+
 /* ---- Distillation loss of the refinement head (App. C.3, Eq. 10) ----
  *
  * The training objective of the corrector on a batch of blocks: at every reached position j

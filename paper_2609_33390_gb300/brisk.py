@@ -80,6 +80,9 @@ _SIGS = [
     ("brisk_acceptance_weights", ctypes.c_int,
      [ctypes.c_int32, _vp, _vp, _vp, ctypes.c_double, _vp, _vp, _vp]),
     ("brisk_tpf_isd", ctypes.c_double, [ctypes.c_int32, ctypes.c_double]),
+    ("brisk_replay_diagnostics", ctypes.c_int,
+     [ctypes.POINTER(Dims), ctypes.POINTER(Params), _vp, _vp, _vp, _vp, _vp, _vp, ctypes.c_int32,
+      _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp]),
     ("brisk_distill_loss", ctypes.c_int,
      [ctypes.POINTER(Dims), _vp, _vp, _vp, _vp, _vp, ctypes.c_float, _vp, _vp, _vp, _vp]),
 ]
@@ -223,6 +226,18 @@ class DecodeTail:
             int(select_mode), int(verify_mode), _p(u_acc), _p(u_res), _p(a), _p(out), _p(corr),
             _p(self.workspace), _stream(stream)), "verify")
         return {"accepted_len": a, "out_tokens": out, "correction": corr}
+
+    def replay(self, block, select_mode=SELECT_GREEDY, stream=None):
+        """Same-state replay diagnostics (App. B, Eq. 6) of one block (see synth.make_block)."""
+        B, L, K = self.B, self.L, self.K
+        head, flags, fb, ref = self._i32(B, L), self._i32(B, L), self._i32(B), self._f32(B, L, K)
+        _check(lib().brisk_replay_diagnostics(
+            ctypes.byref(self.dims), ctypes.byref(self.params), _p(self.tables),
+            _p(block["hidden"]), _p(block["h_c"]), _p(block["x0"]), _p(block["logits_q"]),
+            _p(block["logits_p"]), int(select_mode), _p(block["u_sel"]), _p(block["u_acc"]),
+            _p(head), _p(flags), _p(fb), _p(ref), _p(self.workspace), _stream(stream)),
+            "replay_diagnostics")
+        return {"head_tokens": head, "flags": flags, "first_breaker": fb, "refined": ref}
 
     def distill_loss(self, logits_p, cand_ids, cand_logprob, refined, accepted_len, beta=0.01,
                      with_grad=True, stream=None):

@@ -29,7 +29,7 @@ inline size_t esize(int dt) { return dt == BRISK_DT_BF16 ? 2 : 4; }
 // ---------------------------------------------------------------- workspace layout
 struct WsLayout {
   size_t status, counters, part_val, part_id, part_m, part_s, argmax_p, lse_p;
-  size_t cand_ids, cand_logprob, lse_q, sel, refined, Hm, G, G0, distill, total;
+  size_t cand_ids, cand_logprob, lse_q, sel, refined, Hm, G, G0, distill, base_rank, total;
   int nchunk_q, nchunk_p, KP;   // chunks per proposal row (row layout) and verifier row (split)
 };
 
@@ -60,6 +60,7 @@ WsLayout ws_layout(const brisk_dims* d) {
   w.G = take(sizeof(float) * BL * 2 * S);
   w.G0 = take(sizeof(float) * d->B * S);
   w.distill = take(sizeof(float) * d->B);   // per-sequence loss partials of brisk_distill_loss
+  w.base_rank = take(sizeof(int32_t) * BL);  // base selections of brisk_replay_diagnostics
   w.total = o;
   return w;
 }
@@ -573,6 +574,78 @@ brisk_status brisk_distill_loss(const brisk_dims* d, const void* logits_p, const
   a.arrivals = at<int32_t>(ws, w.status) + 16;   // a word of the (cleared) status block
   a.status = at<int32_t>(ws, w.status);
   BRISK_CUDA(launch_distill(a, st));
+  return BRISK_OK;
+}
+
+brisk_status brisk_replay_diagnostics(const brisk_dims* d, const brisk_params* p, const void* tables,
+                                      const void* hidden, const void* h_ctx, const int32_t* x0,
+                                      const void* logits_q, const void* logits_p,
+                                      int32_t select_mode, const float* u_sel, const float* u_acc,
+                                      int32_t* head_tokens, int32_t* flags,
+                                      int32_t* first_breaker, float* refined, void* ws,
+                                      void* stream) {
+  if (!dims_ok(d) || !params_ok(p) || !tables || !hidden || !h_ctx || !x0 || !logits_q ||
+      !logits_p || !u_acc || !head_tokens || !flags || !first_breaker || !ws ||
+      !aligned(ws, ALIGN) || !aligned(tables, ALIGN) || !aligned(logits_q, esize(d->logits_dtype)) ||
+      !aligned(logits_p, esize(d->logits_dtype)))
+    return BRISK_ERR_INVALID_ARG;
+  if (select_mode != BRISK_SELECT_GREEDY && select_mode != BRISK_SELECT_SAMPLE)
+    return BRISK_ERR_INVALID_ARG;
+  if (select_mode == BRISK_SELECT_SAMPLE && !u_sel) return BRISK_ERR_INVALID_ARG;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const WsLayout w = ws_layout(d);
+  brisk_status s = clear_ws(w, d, ws, st);
+  if (s != BRISK_OK) return s;
+  const int BL = d->B * d->L;
+  int32_t* cand_ids = at<int32_t>(ws, w.cand_ids);
+  float* cand_lp = at<float>(ws, w.cand_logprob);
+  float* ref = refined ? refined : at<float>(ws, w.refined);
+  // candidates, and the verifier rows' log-partition
+  SweepLaunch sq{};
+  sq.seg[0] = make_seg(w, ws, 0, logits_q, BL, d->K, cand_ids, cand_lp, at<float>(ws, w.lse_q));
+  sq.nseg = 1;
+  sq.V = d->V;
+  sq.mode = SWEEP_ROWS;
+  sq.nchunk = w.nchunk_q;
+  sq.KP = w.KP;
+  sq.dtype = d->logits_dtype;
+  sq.status = at<int32_t>(ws, w.status);
+  BRISK_CUDA(launch_sweep(sq, st));
+  SweepLaunch sp = sq;
+  sp.seg[0] = make_seg(w, ws, 1, logits_p, BL, 1, at<int32_t>(ws, w.argmax_p), nullptr,
+                       at<float>(ws, w.lse_p));
+  sp.mode = SWEEP_SPLIT;
+  sp.nchunk = w.nchunk_p;
+  BRISK_CUDA(launch_sweep(sp, st));
+  // the head along the factual base prefix
+  s = hidden_products(d, p, tables, hidden, h_ctx, w, ws, st);
+  if (s != BRISK_OK) return s;
+  ScanArgs a = scan_args(d, p, tables, w, ws);
+  a.select_mode = select_mode;
+  a.do_select = 1;
+  a.logits_q = logits_q;
+  a.cand_ids = cand_ids;
+  a.cand_logprob = cand_lp;
+  a.x0 = x0;
+  a.u_sel = u_sel;
+  a.sel_tokens = head_tokens;
+  a.refined = ref;
+  a.base_prefix = 1;
+  a.base_rank = at<int32_t>(ws, w.base_rank);
+  BRISK_CUDA(launch_scan(a, st));
+  ReplayArgs r{};
+  r.B = d->B; r.L = d->L; r.V = d->V; r.K = d->K; r.logits_dt = d->logits_dtype;
+  r.logits_p = logits_p;
+  r.lse_p = at<float>(ws, w.lse_p);
+  r.cand_ids = cand_ids;
+  r.cand_logprob = cand_lp;
+  r.base_rank = a.base_rank;
+  r.head_tokens = head_tokens;
+  r.u_acc = u_acc;
+  r.flags = flags;
+  r.first_breaker = first_breaker;
+  r.status = at<int32_t>(ws, w.status);
+  BRISK_CUDA(launch_replay(r, st));
   return BRISK_OK;
 }
 

@@ -264,6 +264,10 @@ struct ScanArgs {
   const float* Fh;       // [S, 5]
   const float* wg;       // [S + 5]
   float b_g, alpha;
+  // same-state replay (App. B): feed the base selection forward instead of the head's, and
+  // record its rank
+  int base_prefix;
+  int32_t* base_rank;    // [B, L] (base_prefix only)
   // select outputs (or verify inputs when do_select == 0)
   int32_t* sel_tokens;   // [B, L]
   float* refined;        // [B, L, K]
@@ -296,6 +300,22 @@ struct DistillArgs {
   int32_t* status;
 };
 cudaError_t launch_distill(const DistillArgs& a, cudaStream_t stream);
+
+// ---------------------------------------------------------------- same-state replay
+struct ReplayArgs {
+  int B, L, V, K, logits_dt;
+  const void* logits_p;        // [B, L, V]
+  const float* lse_p;          // [B, L]
+  const int32_t* cand_ids;     // [B, L, K]
+  const float* cand_logprob;   // [B, L, K]
+  const int32_t* base_rank;    // [B, L]
+  const int32_t* head_tokens;  // [B, L]
+  const float* u_acc;          // [B, L]
+  int32_t* flags;              // [B, L]
+  int32_t* first_breaker;      // [B]
+  int32_t* status;
+};
+cudaError_t launch_replay(const ReplayArgs& a, cudaStream_t stream);
 
 size_t scan_smem_bytes(int L, int K, int S, int V);
 cudaError_t launch_scan(const ScanArgs& a, cudaStream_t stream);

@@ -719,12 +719,20 @@ corrector_kernel(const __grid_constant__ ScanArgs a) {
     const float gamma = sig_alpha * sigmoid_fast(gate);
     const float dk = __shfl_sync(FULL_MASK, r, (lane * LSTEP) & 31);
     const float ref = lane < K ? sm.clp[i * K + lane] + gamma * dk : -INFINITY;
+    const float u_cur_draw = u_cur;
     const int pick = select_warp(ref, K, a.select_mode, u_cur);
     if (warp == 0 && lane < K) a.refined[(bL + i) * K + lane] = ref;
     if (a.select_mode == BRISK_SELECT_SAMPLE && i + 1 < L) u_cur = a.u_sel[bL + i + 1];
-    prank = pick;
-    prev = ci[pick];
-    if (tid == 0) a.sel_tokens[bL + i] = prev;
+    if (tid == 0) a.sel_tokens[bL + i] = ci[pick];
+    // the token fed forward: the head's selection, or in a same-state replay the base
+    // selection (the Select rule on the base scores log q, same draw)
+    int fwd = pick;
+    if (a.base_prefix) {
+      fwd = select_warp(lane < K ? sm.clp[i * K + lane] : -INFINITY, K, a.select_mode, u_cur_draw);
+      if (tid == 0) a.base_rank[bL + i] = fwd;
+    }
+    prank = fwd;
+    prev = ci[fwd];
     // advance the pipeline
     if (i + 1 < L) {
       if constexpr (PIPE) {
