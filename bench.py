@@ -409,6 +409,7 @@ def run_ours(args):
 
     if rank != 0:
         return 0
+    graph_loop = run_graph_loop(dev)
     cpu = None
     if not args.no_cpu_baseline:
         cpu = cpu_baseline_entry(list(range(CPU_SAMPLE_SEQS)))
@@ -441,6 +442,7 @@ def run_ours(args):
                                "positions_shown": min(8, wl.L),
                                "tpf_unit_cost": prof_tpf,
                                "w_bar": [round(x, 4) for x in prof_w[:8]]},
+        "graph_loop": graph_loop,
         "distill_loss_us": distill_us,
         "replay": {"first_breakers": n_fb,
                    "intervention_rate_at_breakers": n_int / max(1, n_fb),
@@ -453,6 +455,49 @@ def run_ours(args):
         import torch.distributed as dist
         dist.destroy_process_group()
     return 0
+
+
+def run_graph_loop(dev, blocks=30):
+    """Per-block latency of the decode tail on one sequence (the `single` workload), as direct
+    calls and as replays of the captured CUDA graph (App. F), anchors chained on the device."""
+    import torch
+    from paper_2609_33390_gb300 import brisk, synth
+    wl = synth.WORKLOADS["single"]
+    tail = brisk.DecodeTail.for_workload(wl, synth.make_weights(wl, dev), dev)
+    tail.prepare()
+    blk = synth.make_block(wl, dev)
+    sm, vm = brisk.mode_ids(wl.select_mode, wl.verify_mode)
+    stream = torch.cuda.Stream()
+    out = tail.alloc_outputs(full=False)
+    anchor = blk["x0"].clone()
+    out["next_anchor"] = anchor
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        for _ in range(5):
+            tail.tail(blk, sm, vm, out=out, x0=anchor, stream=stream)
+        e0.record(stream)
+        for _ in range(blocks):
+            tail.tail(blk, sm, vm, out=out, x0=anchor, stream=stream)
+        e1.record(stream)
+    stream.synchronize()
+    direct_us = 1000.0 * e0.elapsed_time(e1) / blocks
+    g = tail.graph(blk, sm, vm, stream=stream)
+    with torch.cuda.stream(stream):
+        for _ in range(5):
+            g.launch()
+        e0.record(stream)
+        acc = 0
+        for _ in range(blocks):
+            g.launch()
+        e1.record(stream)
+    stream.synchronize()
+    graph_us = 1000.0 * e0.elapsed_time(e1) / blocks
+    acc = int(g.out["accepted_len"].sum())
+    g.close()
+    return {"workload": "single", "B": wl.B, "L": wl.L, "V": wl.V, "blocks": blocks,
+            "direct_us_per_block": direct_us, "graph_us_per_block": graph_us,
+            "kernels_per_block": brisk.kernels_per_tail(tail.dims),
+            "accepted_last_block": acc}
 
 
 def run_e2e(args, tail, pool, wl, sm, vm, dev):

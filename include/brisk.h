@@ -210,6 +210,25 @@ brisk_status brisk_decode_tail(const brisk_dims *dims, const brisk_params *param
                                int32_t verify_mode, void *workspace, const brisk_events *ev,
                                void *stream);
 
+/* ---- The decode tail as a replayable CUDA graph (App. F: fused head plus CUDA Graph replay) ----
+ *
+ * brisk_tail_graph_create makes one direct brisk_decode_tail call with these arguments (it
+ * checks them and prepares the library's side streams), then captures a second call on
+ * `stream` (a non-default stream, thread-local capture) into a graph whose launches read and
+ * write exactly the buffers of `io`, `tables` and `workspace`. brisk_tail_graph_launch replays
+ * it on `stream`: refresh the inputs in place between launches; with io->x0 == io->next_anchor
+ * the anchor of block t+1 is the last committed token of block t, on the device. The buffers
+ * must outlive the graph; the graph and the workspace must not be used by overlapping launches.
+ * Returns the status of the direct call, BRISK_ERR_INVALID_ARG for a NULL out/stream, or
+ * BRISK_ERR_CUDA if capture or instantiation fails. */
+typedef struct brisk_graph brisk_graph;
+brisk_status brisk_tail_graph_create(const brisk_dims *dims, const brisk_params *params,
+                                     const void *tables, const brisk_tail_io *io,
+                                     int32_t select_mode, int32_t verify_mode, void *workspace,
+                                     void *stream, brisk_graph **out);
+brisk_status brisk_tail_graph_launch(brisk_graph *graph, void *stream);
+void brisk_tail_graph_destroy(brisk_graph *graph);
+
 /* Kernels one brisk_decode_tail call launches for `dims` (0 if dims are invalid). */
 int32_t brisk_kernels_per_tail(const brisk_dims *dims);
 

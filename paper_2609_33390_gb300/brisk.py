@@ -80,6 +80,11 @@ _SIGS = [
     ("brisk_acceptance_weights", ctypes.c_int,
      [ctypes.c_int32, _vp, _vp, _vp, ctypes.c_double, _vp, _vp, _vp]),
     ("brisk_tpf_isd", ctypes.c_double, [ctypes.c_int32, ctypes.c_double]),
+    ("brisk_tail_graph_create", ctypes.c_int,
+     [ctypes.POINTER(Dims), ctypes.POINTER(Params), _vp, ctypes.POINTER(TailIO), ctypes.c_int32,
+      ctypes.c_int32, _vp, _vp, ctypes.POINTER(_vp)]),
+    ("brisk_tail_graph_launch", ctypes.c_int, [_vp, _vp]),
+    ("brisk_tail_graph_destroy", None, [_vp]),
     ("brisk_replay_diagnostics", ctypes.c_int,
      [ctypes.POINTER(Dims), ctypes.POINTER(Params), _vp, _vp, _vp, _vp, _vp, _vp, ctypes.c_int32,
       _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp]),
@@ -260,17 +265,21 @@ class DecodeTail:
                      lse_q=self._f32(B, L), sel_tokens=self._i32(B, L), refined=self._f32(B, L, K))
         return o
 
+    @staticmethod
+    def _io(block, out, x0):
+        return TailIO(_p(block["logits_q"]), _p(block["logits_p"]), _p(block["hidden"]),
+                      _p(block["h_c"]), _p(block["x0"] if x0 is None else x0), _p(block.get("u_sel")),
+                      _p(block.get("u_acc")), _p(block.get("u_res")), _p(out.get("cand_ids")),
+                      _p(out.get("cand_logprob")), _p(out.get("lse_q")), _p(out.get("sel_tokens")),
+                      _p(out.get("refined")), _p(out["accepted_len"]), _p(out["out_tokens"]),
+                      _p(out["correction"]), _p(out.get("next_anchor")))
+
     def tail(self, block, select_mode=SELECT_GREEDY, verify_mode=VERIFY_GREEDY, out=None, x0=None,
              events=None, stream=None):
         """One fused decode-tail call on the tensors of ``block`` (see ``synth.make_block``)."""
         if out is None:
             out = self.alloc_outputs()
-        io = TailIO(_p(block["logits_q"]), _p(block["logits_p"]), _p(block["hidden"]),
-                    _p(block["h_c"]), _p(block["x0"] if x0 is None else x0), _p(block.get("u_sel")),
-                    _p(block.get("u_acc")), _p(block.get("u_res")), _p(out.get("cand_ids")),
-                    _p(out.get("cand_logprob")), _p(out.get("lse_q")), _p(out.get("sel_tokens")),
-                    _p(out.get("refined")), _p(out["accepted_len"]), _p(out["out_tokens"]),
-                    _p(out["correction"]), _p(out.get("next_anchor")))
+        io = self._io(block, out, x0)
         ev = None
         if events is not None:
             ev = ctypes.byref(Events(*[_vp(e.cuda_event) for e in events]))
@@ -280,8 +289,60 @@ class DecodeTail:
                "decode_tail")
         return out
 
+    def graph(self, block, select_mode=SELECT_GREEDY, verify_mode=VERIFY_GREEDY, out=None,
+              chain_anchor=True, stream=None):
+        """The decode tail on these buffers captured into a replayable CUDA graph (App. F). With
+        chain_anchor the anchor buffer is also the next-anchor output, so replays chain blocks."""
+        return TailGraph(self, block, select_mode, verify_mode, out, chain_anchor, stream)
+
     def device_status(self, clear=True, stream=None) -> int:
         return int(lib().brisk_last_device_status(_p(self.workspace), int(clear), _stream(stream)))
+
+
+class TailGraph:
+    """A captured decode tail (see brisk_tail_graph_create); launch() replays it."""
+
+    def __init__(self, tail, block, select_mode, verify_mode, out, chain_anchor, stream):
+        if stream is None:
+            raise ValueError("capture needs a non-default stream")
+        self.tail = tail
+        self.block = block
+        self.out = tail.alloc_outputs() if out is None else out
+        if chain_anchor:
+            self.anchor = block["x0"].clone()
+            self.out["next_anchor"] = self.anchor
+        else:
+            self.anchor = block["x0"]
+        self.stream = stream
+        self._iob = tail._io(block, self.out, self.anchor)
+        saved = self.anchor.clone()
+        torch.cuda.synchronize()
+        h = _vp()
+        _check(lib().brisk_tail_graph_create(ctypes.byref(tail.dims), ctypes.byref(tail.params),
+                                             _p(tail.tables), ctypes.byref(self._iob),
+                                             int(select_mode), int(verify_mode),
+                                             _p(tail.workspace), _stream(stream), ctypes.byref(h)),
+               "tail_graph_create")
+        self.handle = h
+        # the direct call inside create advanced a chained anchor: start the replays from x0
+        with torch.cuda.stream(stream):
+            self.anchor.copy_(saved)
+        stream.synchronize()
+
+    def launch(self):
+        _check(lib().brisk_tail_graph_launch(self.handle, _stream(self.stream)), "tail_graph_launch")
+        return self.out
+
+    def close(self):
+        if self.handle:
+            lib().brisk_tail_graph_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
 
 
 def mode_ids(select_mode: str, verify_mode: str):
