@@ -72,8 +72,12 @@ def measured_peaks():
 
 
 def sweep_source_hash() -> str:
-    with open(SWEEP_KERNEL_SRC, "rb") as f:
-        return hashlib.sha1(f.read()).hexdigest()[:12]
+    """Hash of the sweep source's code: line comments, trailing blanks and empty lines are left
+    out, so that an edit of the comments alone keeps a traffic record that is still valid."""
+    with open(SWEEP_KERNEL_SRC) as f:
+        lines = [ln.split("//", 1)[0].rstrip() for ln in f]
+    code = "\n".join(ln for ln in lines if ln)
+    return hashlib.sha1(code.encode()).hexdigest()[:12]
 
 
 def recorded_traffic(workload: str):

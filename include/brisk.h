@@ -50,7 +50,7 @@ typedef enum brisk_status {
   BRISK_ERR_UNSUPPORTED = 2,   /* valid request this build does not implement                   */
   BRISK_ERR_CUDA = 3,          /* a CUDA call or kernel launch failed                           */
   BRISK_ERR_TIMEOUT = 4,       /* a bounded device-side wait gave up                            */
-  BRISK_ERR_NUMERIC = 5        /* a row's log-partition was not finite (NaN / all -inf)          */
+  BRISK_ERR_NUMERIC = 5        /* a non-finite log-partition (NaN / all -inf) or a NaN score     */
 } brisk_status;
 
 typedef enum brisk_dtype { BRISK_DT_F32 = 0, BRISK_DT_BF16 = 1 } brisk_dtype;
@@ -235,7 +235,8 @@ int32_t brisk_kernels_per_tail(const brisk_dims *dims);
 /* Reads the device status word of `workspace` (synchronises `stream`): BRISK_OK or the first
  * device-side problem recorded by the most recent call on this workspace (every call clears the
  * word when it starts). Device-side problems: a non-finite log-partition or a candidate id that
- * a row with no finite logit left out of range (BRISK_ERR_NUMERIC); an anchor or selected token
+ * a row with no finite logit left out of range, or a NaN refined score (BRISK_ERR_NUMERIC; Select
+ * then ranks NaN below every number, so the selection is still a candidate); an anchor or selected token
  * outside [0, V) (BRISK_ERR_INVALID_ARG; the id is replaced by 0 so that nothing reads out of
  * bounds). With clear != 0 the word is reset to BRISK_OK afterwards. */
 brisk_status brisk_last_device_status(void *workspace, int32_t clear, void *stream);

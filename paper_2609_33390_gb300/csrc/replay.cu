@@ -36,7 +36,7 @@ replay_kernel(const __grid_constant__ ReplayArgs a) {
     int rh = -1;
     for (int k = 0; k < K; ++k)
       if (a.cand_ids[row * K + k] == xh) { rh = k; break; }
-    if (rh < 0 || xb < 0 || xb >= a.V) { set_status(a.status, BRISK_ERR_INVALID_ARG); continue; }
+    if (rh < 0 || xb < 0 || xb >= a.V || xh < 0 || xh >= a.V) { set_status(a.status, BRISK_ERR_INVALID_ARG); continue; }
     const float lse = a.lse_p[row];
     const float u = a.u_acc[row];
     // alpha = min(1, p(x) / q(x)) = min(1, exp(log p(x) - log q(x)))

@@ -104,8 +104,10 @@ __device__ __forceinline__ float load_logit(const void* base, int dt, size_t idx
 __device__ __forceinline__ int select_warp(float ref, int K, int mode, float u) {
   const int lane = threadIdx.x & 31;
   if (mode == BRISK_SELECT_GREEDY) {
-    float bv = ref;
-    int bk = lane < K ? lane : 0x7fffffff;
+    // a NaN score ranks as -inf, so the comparisons below order every lane and all lanes
+    // agree on one rank in [0, K) whatever the scores hold
+    float bv = (lane < K && !isnan(ref)) ? ref : -INFINITY;
+    int bk = lane < K ? lane : K;
 #pragma unroll
     for (int off = 16; off; off >>= 1) {
       const float ov = __shfl_xor_sync(FULL_MASK, bv, off);
@@ -721,7 +723,11 @@ corrector_kernel(const __grid_constant__ ScanArgs a) {
     const float ref = lane < K ? sm.clp[i * K + lane] + gamma * dk : -INFINITY;
     const float u_cur_draw = u_cur;
     const int pick = select_warp(ref, K, a.select_mode, u_cur);
-    if (warp == 0 && lane < K) a.refined[(bL + i) * K + lane] = ref;
+    if (warp == 0) {
+      if (lane < K) a.refined[(bL + i) * K + lane] = ref;
+      if (__any_sync(FULL_MASK, lane < K && isnan(ref)) && lane == 0)
+        set_status(a.status, BRISK_ERR_NUMERIC);
+    }
     if (a.select_mode == BRISK_SELECT_SAMPLE && i + 1 < L) u_cur = a.u_sel[bL + i + 1];
     if (tid == 0) a.sel_tokens[bL + i] = ci[pick];
     // the token fed forward: the head's selection, or in a same-state replay the base

@@ -30,14 +30,14 @@ def _to(d, device):
     return {k: (v.to(device) if torch.is_tensor(v) else v) for k, v in d.items()}
 
 
-def _run_and_check(B, wl, weights, block, seqs=None, unfused=True):
+def _run_and_check(B, wl, weights, block, seqs=None, unfused=True, status=None):
     dev = torch.device("cuda")
     sm, vm = B.mode_ids(wl.select_mode, wl.verify_mode)
     tail = B.DecodeTail.for_workload(wl, weights, dev, B=block["logits_q"].shape[0])
     tail.prepare()
     out = tail.tail(block, sm, vm)
     torch.cuda.synchronize()
-    assert tail.device_status() == B.OK
+    assert tail.device_status() == (B.OK if status is None else status)
     g = to_numpy(out)
     if unfused:
         c = tail.topk(block["logits_q"])
@@ -115,7 +115,9 @@ def test_ties_and_minus_infinity(brisk):
     lq[1, 2] = torch.round(lq[1, 2].float() * 2).to(lq.dtype)   # many exact ties
     lq[1, 3, :] = float("-inf")
     lq[1, 3, 500:503] = 2.0                    # three finite values, the rest -inf
-    rep, g = _run_and_check(brisk, wl, weights, block)
+    # the last row's top1-top4 gap is +inf, so its gate and refined scores are NaN: reported
+    rep, g = _run_and_check(brisk, wl, weights, block, status=brisk.ERR_NUMERIC)
+    assert np.isnan(g["refined"][1, 3]).all() and np.isfinite(g["refined"][:, :3]).all()
     assert list(g["cand_ids"][0, 0]) == list(range(wl.K))
     assert list(g["cand_ids"][1, 3, :3]) == [500, 501, 502]
 
@@ -144,6 +146,46 @@ def test_non_finite_row_sets_numeric_status(brisk):
     torch.cuda.synchronize()
     assert tail.device_status() == brisk.ERR_NUMERIC
     assert tail.device_status() == brisk.OK   # cleared by the first read
+
+
+@pytest.mark.parametrize("mode", ["greedy", "sample"])
+def test_nan_scores_still_select_a_candidate(brisk, mode):
+    """NaN candidate log-probabilities (caller data, or a row with no finite logit) give NaN
+    refined scores: Select ranks them below every number, every selection is still one of the
+    position's candidates and the device status reports the numeric problem."""
+    wl = synth.Workload("nansel", B=3, L=6, V=1024, d=32, K=8, r=16)
+    weights = _to(synth.make_weights(wl, "cpu"), "cuda")
+    block = _to(synth.make_block(wl, "cpu"), "cuda")
+    tail = brisk.DecodeTail.for_workload(wl, weights)
+    tail.prepare()
+    c = tail.topk(block["logits_q"])
+    torch.cuda.synchronize()
+    assert tail.device_status() == brisk.OK
+    lp = c["cand_logprob"].clone()
+    lp[0, 2, :] = float("nan")          # a whole position
+    lp[1, :, 0] = float("nan")          # rank 0 everywhere
+    lp[2, 4, 3:] = float("nan")         # part of a position
+    sm = brisk.SELECT_SAMPLE if mode == "sample" else brisk.SELECT_GREEDY
+    s = tail.select(block["hidden"], block["h_c"], block["x0"], block["logits_q"], c["cand_ids"],
+                    lp, sm, u_sel=block["u_sel"])
+    torch.cuda.synchronize()
+    assert tail.device_status() == brisk.ERR_NUMERIC
+    sel = s["sel_tokens"].cpu()
+    ids = c["cand_ids"].cpu()
+    assert bool((sel[..., None] == ids).any(-1).all())
+    if mode == "greedy":
+        # rows without NaN keep the argmax of the finite scores
+        ref = s["refined"].cpu()
+        for b, i in ((1, 0), (2, 4)):
+            r = ref[b, i].clone()
+            r[torch.isnan(r)] = float("-inf")
+            assert int(sel[b, i]) == int(ids[b, i, int(torch.argmax(r))])
+    v = tail.verify(block["logits_p"], s["sel_tokens"], c["cand_ids"], s["refined"], sm,
+                    brisk.VERIFY_GREEDY)
+    torch.cuda.synchronize()
+    assert tail.device_status() == brisk.OK
+    a = v["accepted_len"].cpu()
+    assert bool(((a >= 0) & (a <= wl.L)).all())
 
 
 def test_generator_same_on_cpu_and_gpu():
