@@ -119,8 +119,8 @@ typedef struct brisk_tail_io {
 } brisk_tail_io;
 
 /* Optional timing hooks: cudaEvent_t handles (as void*) recorded right before and right after
- * the two vocabulary-sweep kernels of brisk_decode_tail (proposal rows on `stream`, verifier
- * rows on the library's side stream). NULL fields are skipped. */
+ * the two vocabulary-sweep kernels of brisk_decode_tail, each on the stream that kernel runs on
+ * (the two launches may overlap). NULL fields are skipped. */
 typedef struct brisk_events {
   void *sweep_q_begin, *sweep_q_end, *sweep_p_begin, *sweep_p_end;
 } brisk_events;
@@ -196,13 +196,15 @@ brisk_status brisk_verify_block(const brisk_dims *dims, const void *logits_p,
                                 int32_t *out_tokens, int32_t *correction, void *workspace,
                                 void *stream);
 
-/* Steps 1-3 for one block step (Algorithm 1(b) lines after the backbone pass): the same results,
- * bit for bit, as brisk_topk_candidates + brisk_corrector_select + brisk_verify_block on the same
- * inputs. The corrector needs only the proposal candidates, so the verifier rows are swept on a
- * library side stream while the corrector runs (and the hidden-state products run on another
- * side stream during the proposal sweep); the call still only enqueues work and the results are
- * ordered on `stream` (the side streams fork from and join back to it, also under graph
- * capture). The first call on a device creates the side streams and their events: make it
+/* Steps 1-3 for one block step (the steps of Algorithm 1(b) after the backbone pass): the same
+ * results, bit for bit, as brisk_topk_candidates + brisk_corrector_select + brisk_verify_block on
+ * the same inputs. The work runs on library side streams of decreasing priority: the
+ * hidden-state products; the proposal sweep, corrector and verification (the critical path);
+ * the verifier-row sweep, which starts at once and fills the SMs the others leave free. When the
+ * batch is small enough that the proposal rows are swept in several chunks each, the critical
+ * path runs on `stream` itself and the verifier sweep starts after the proposal sweep. The call
+ * only enqueues work and the results are ordered on `stream` (the side streams fork from and
+ * join back to it, also under graph capture). The first call on a device creates the side streams and their events: make it
  * before any stream capture. Calls from several host threads are serialised while they enqueue.
  * `ev` may be NULL. */
 brisk_status brisk_decode_tail(const brisk_dims *dims, const brisk_params *params,

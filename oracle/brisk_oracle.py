@@ -203,7 +203,7 @@ def corrector_sequence(p: Params, hidden: np.ndarray, h_c: np.ndarray, x0: int,
                        u_sel: Optional[np.ndarray] = None,
                        force: Optional[Dict[int, int]] = None,
                        prefix_ranks: Optional[np.ndarray] = None) -> CorrectorTrace:
-    """Algorithm 1(b) lines for i = 1..M of one sequence (0-based i here).
+    """The corrector loop of Algorithm 1(b) over i = 1..M for one sequence (0-based i here).
 
     hidden: [L, d] MASK hidden states m_i; h_c: [d]; x0: anchor token;
     rows_q(i): proposal logit row i; cand_ids/cand_logprob: [L, K] from step 1;

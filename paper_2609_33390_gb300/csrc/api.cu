@@ -149,11 +149,15 @@ SweepSeg make_seg(const WsLayout& w, void* ws, int seg, const void* logits, int 
 // G = Hm[:BL] [W_z[:, :r] ; W_h[:, :r]]^T and G0 = Hm[BL:] W0[:, :r]^T. With bf16 weights the
 // products run on the tensor cores: the first one writes Hm as three bf16 parts, which the
 // second one multiplies by the weight blocks written three times along k (fp32-level accuracy).
-// The first product (k = d long, few 256-wide tiles) uses 64-wide tiles and a 4-deep pipeline:
-// four times the CTAs, each streaming a quarter of the weights.
+// The first product (k = d long) has few 128-row tiles for small batches: there it uses 64-wide
+// column tiles and a 4-deep pipeline (four times the CTAs, each streaming a quarter of the
+// weights). With `wide` (large batches, the products running beside the proposal sweep) it uses
+// 256-wide tiles and a 2-deep pipeline: a quarter of the CTAs, so the sweep waits for fewer SMs,
+// and the hidden states are read once. Tile width does not change any product's summation
+// order, so both give the same bits.
 brisk_status hidden_products(const brisk_dims* d, const brisk_params* p, const void* tables,
                              const void* hidden, const void* h_ctx, const WsLayout& w, void* ws,
-                             cudaStream_t st) {
+                             cudaStream_t st, bool wide) {
   const TbLayout t = tb_layout(d);
   const int BL = d->B * d->L, r = d->r, S = 2 * d->r, hd = d->hidden_dtype;
   int32_t* status = at<int32_t>(ws, w.status);
@@ -161,10 +165,11 @@ brisk_status hidden_products(const brisk_dims* d, const brisk_params* p, const v
       aligned(h_ctx, 16)) {
     __nv_bfloat16* Hs = at<__nv_bfloat16>(ws, w.Hm);   // [BL + B, 3r]: hi | mid | lo
     const int r3 = 3 * r;
+    const int bn = wide ? 256 : 64;
     const TcSpec first[2] = {
-        {BL, r, d->d, hidden, d->d, p->P_h, d->d, 1, Hs, r3, nullptr, 0, 64},
-        {d->B, r, d->d, h_ctx, d->d, p->P_h, d->d, 1, Hs + (size_t)BL * r3, r3, nullptr, 0, 64}};
-    BRISK_CUDA(gemm_tc_grouped(first, 2, status, st, 4));
+        {BL, r, d->d, hidden, d->d, p->P_h, d->d, 1, Hs, r3, nullptr, 0, bn},
+        {d->B, r, d->d, h_ctx, d->d, p->P_h, d->d, 1, Hs + (size_t)BL * r3, r3, nullptr, 0, bn}};
+    BRISK_CUDA(gemm_tc_grouped(first, 2, status, st, wide ? 2 : 4));
     const TcSpec second[2] = {
         {BL, 2 * S, r3, Hs, r3, at<__nv_bfloat16>(tables, t.W2s), r3, 0, at<float>(ws, w.G), 2 * S,
          nullptr, 0, 0},
@@ -187,9 +192,10 @@ brisk_status hidden_products(const brisk_dims* d, const brisk_params* p, const v
 // A side stream per device (created on the first fused call on that device) and the events that
 // fork work onto it and join it back, so that one call can run independent stages concurrently.
 struct SideStream {
-  cudaStream_t hi = nullptr;   // highest priority: the hidden-state products
-  cudaStream_t lo = nullptr;   // lowest priority: the verifier-row sweep
-  cudaEvent_t ev[4] = {nullptr, nullptr, nullptr, nullptr};
+  cudaStream_t hi = nullptr;    // highest priority: the hidden-state products
+  cudaStream_t mid = nullptr;   // middle priority: proposal sweep, corrector, verification
+  cudaStream_t lo = nullptr;    // lowest priority: the verifier-row sweep
+  cudaEvent_t ev[5] = {};
 };
 constexpr int MAX_DEVICES = 256;
 std::mutex g_side_mu;
@@ -202,13 +208,16 @@ SideStream* side_stream() {
   if (!ss.hi) {
     int least = 0, greatest = 0;
     if (cudaDeviceGetStreamPriorityRange(&least, &greatest) != cudaSuccess) return nullptr;
-    cudaStream_t hi = nullptr, lo = nullptr;
+    cudaStream_t hi = nullptr, mid = nullptr, lo = nullptr;
     if (cudaStreamCreateWithPriority(&hi, cudaStreamNonBlocking, greatest) != cudaSuccess ||
+        cudaStreamCreateWithPriority(&mid, cudaStreamNonBlocking, (least + greatest) / 2) !=
+            cudaSuccess ||
         cudaStreamCreateWithPriority(&lo, cudaStreamNonBlocking, least) != cudaSuccess)
       return nullptr;
     for (auto& e : ss.ev)
       if (cudaEventCreateWithFlags(&e, cudaEventDisableTiming) != cudaSuccess) return nullptr;
     ss.lo = lo;
+    ss.mid = mid;
     ss.hi = hi;
   }
   return &ss;
@@ -357,7 +366,7 @@ brisk_status brisk_corrector_select(const brisk_dims* d, const brisk_params* p, 
   const WsLayout w = ws_layout(d);
   brisk_status s = clear_ws(w, d, ws, st);
   if (s != BRISK_OK) return s;
-  s = hidden_products(d, p, tables, hidden, h_ctx, w, ws, st);
+  s = hidden_products(d, p, tables, hidden, h_ctx, w, ws, st, false);
   if (s != BRISK_OK) return s;
   ScanArgs a = scan_args(d, p, tables, w, ws);
   a.select_mode = select_mode;
@@ -448,20 +457,30 @@ brisk_status brisk_decode_tail(const brisk_dims* d, const brisk_params* p, const
   int32_t* sel = io->sel_tokens ? io->sel_tokens : at<int32_t>(ws, w.sel);
   float* refined = io->refined ? io->refined : at<float>(ws, w.refined);
 
-  // Schedule. A = the caller's stream, H / W = side streams of highest / lowest priority:
-  //   H: hidden-state products --------.
-  //   A: proposal-row sweep ----------- join -> corrector scan ---- join -> verification
-  //   W:                      `-> verifier-row sweep ----------------'
-  // The corrector needs only the proposal candidates and the hidden products; the verifier rows
-  // are needed only by the verification, so the corrector runs while the verifier rows are
-  // swept. Priorities decide which ready blocks the GPU places first: the products before the
-  // proposal sweep, the corrector before the verifier sweep (which fills the remaining room).
+  // Schedule on side streams forked from the caller's stream A, by priority:
+  //   H (highest): hidden products -----.
+  //   M (middle) : proposal sweep ---- join -> corrector --- join -> verification -> join A
+  //   W (lowest) : verifier sweep ---------------------------'
+  // The block scheduler places ready blocks of higher priority first. The products take their
+  // SMs first; the proposal sweep, on the critical path (proposal candidates -> corrector ->
+  // verification), takes the rest; the verifier sweep, needed only by the verification, starts
+  // at once but only fills room the other two leave: the proposal sweep's ragged end (one
+  // long task per row, ending over tens of microseconds) and the SMs beside the corrector.
+  // In this mode the products use wide tiles (fewer SMs held at the start).
+  // With chunked proposal rows (few rows) the short tasks end together: then the critical path
+  // stays on A and the verifier sweep starts after the proposal sweep, beside the corrector,
+  // which saves the extra fork and keeps the SMs free for the corrector's start; the products,
+  // on the critical path there, use narrow tiles (more CTAs).
+  const bool overlap = w.nchunk_q == 1;
   std::lock_guard<std::mutex> lock(g_side_mu);
   SideStream* ss = side_stream();
   if (!ss) return BRISK_ERR_CUDA;
+  cudaStream_t m = overlap ? ss->mid : st;
   BRISK_CUDA(cudaEventRecord(ss->ev[0], st));
   BRISK_CUDA(cudaStreamWaitEvent(ss->hi, ss->ev[0], 0));
-  s = hidden_products(d, p, tables, io->hidden, io->h_ctx, w, ws, ss->hi);
+  if (overlap) BRISK_CUDA(cudaStreamWaitEvent(m, ss->ev[0], 0));
+  BRISK_CUDA(cudaStreamWaitEvent(ss->lo, ss->ev[0], 0));
+  s = hidden_products(d, p, tables, io->hidden, io->h_ctx, w, ws, ss->hi, overlap);
   if (s != BRISK_OK) return s;
   BRISK_CUDA(cudaEventRecord(ss->ev[1], ss->hi));
 
@@ -479,20 +498,22 @@ brisk_status brisk_decode_tail(const brisk_dims* d, const brisk_params* p, const
                        at<float>(ws, w.lse_p));
   sp.mode = SWEEP_SPLIT;
   sp.nchunk = w.nchunk_p;
-  if (ev && ev->sweep_q_begin) BRISK_CUDA(cudaEventRecord(static_cast<cudaEvent_t>(ev->sweep_q_begin), st));
-  BRISK_CUDA(launch_sweep(sq, st));
-  if (ev && ev->sweep_q_end) BRISK_CUDA(cudaEventRecord(static_cast<cudaEvent_t>(ev->sweep_q_end), st));
-  BRISK_CUDA(cudaEventRecord(ss->ev[2], st));
+  if (ev && ev->sweep_q_begin) BRISK_CUDA(cudaEventRecord(static_cast<cudaEvent_t>(ev->sweep_q_begin), m));
+  BRISK_CUDA(launch_sweep(sq, m));
+  if (ev && ev->sweep_q_end) BRISK_CUDA(cudaEventRecord(static_cast<cudaEvent_t>(ev->sweep_q_end), m));
+  if (!overlap) {
+    BRISK_CUDA(cudaEventRecord(ss->ev[2], m));
+    BRISK_CUDA(cudaStreamWaitEvent(ss->lo, ss->ev[2], 0));
+  }
 
-  // verifier rows on the low-priority stream, after the proposal sweep
-  BRISK_CUDA(cudaStreamWaitEvent(ss->lo, ss->ev[2], 0));
+  // verifier rows on the low-priority stream
   if (ev && ev->sweep_p_begin) BRISK_CUDA(cudaEventRecord(static_cast<cudaEvent_t>(ev->sweep_p_begin), ss->lo));
   BRISK_CUDA(launch_sweep(sp, ss->lo));
   if (ev && ev->sweep_p_end) BRISK_CUDA(cudaEventRecord(static_cast<cudaEvent_t>(ev->sweep_p_end), ss->lo));
   BRISK_CUDA(cudaEventRecord(ss->ev[3], ss->lo));
 
-  // the corrector on the caller's stream, once the hidden products are done
-  BRISK_CUDA(cudaStreamWaitEvent(st, ss->ev[1], 0));
+  // the corrector once the proposal candidates and the hidden products are done
+  BRISK_CUDA(cudaStreamWaitEvent(m, ss->ev[1], 0));
   ScanArgs a = scan_args(d, p, tables, w, ws);
   a.select_mode = select_mode;
   a.verify_mode = verify_mode;
@@ -505,8 +526,8 @@ brisk_status brisk_decode_tail(const brisk_dims* d, const brisk_params* p, const
   a.u_sel = io->u_sel;
   a.sel_tokens = sel;
   a.refined = refined;
-  BRISK_CUDA(launch_scan(a, st));
-  BRISK_CUDA(cudaStreamWaitEvent(st, ss->ev[3], 0));
+  BRISK_CUDA(launch_scan(a, m));
+  BRISK_CUDA(cudaStreamWaitEvent(m, ss->ev[3], 0));
 
   ScanArgs v = scan_args(d, nullptr, nullptr, w, ws);
   v.select_mode = select_mode;
@@ -523,7 +544,11 @@ brisk_status brisk_decode_tail(const brisk_dims* d, const brisk_params* p, const
   v.out_tokens = io->out_tokens;
   v.correction = io->correction;
   v.next_anchor = io->next_anchor;
-  BRISK_CUDA(launch_scan(v, st));
+  BRISK_CUDA(launch_scan(v, m));
+  if (overlap) {
+    BRISK_CUDA(cudaEventRecord(ss->ev[4], m));
+    BRISK_CUDA(cudaStreamWaitEvent(st, ss->ev[4], 0));
+  }
   return BRISK_OK;
 }
 
@@ -618,7 +643,7 @@ brisk_status brisk_replay_diagnostics(const brisk_dims* d, const brisk_params* p
   sp.nchunk = w.nchunk_p;
   BRISK_CUDA(launch_sweep(sp, st));
   // the head along the factual base prefix
-  s = hidden_products(d, p, tables, hidden, h_ctx, w, ws, st);
+  s = hidden_products(d, p, tables, hidden, h_ctx, w, ws, st, false);
   if (s != BRISK_OK) return s;
   ScanArgs a = scan_args(d, p, tables, w, ws);
   a.select_mode = select_mode;

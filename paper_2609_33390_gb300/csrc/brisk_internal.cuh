@@ -6,6 +6,9 @@
 #include <stdint.h>
 #include <math.h>
 #include <atomic>
+#include <mutex>
+#include <utility>
+#include <vector>
 
 #include "../../include/brisk.h"
 
@@ -150,22 +153,30 @@ __device__ __forceinline__ void warp_lse_combine(float& m, float& s) {
 constexpr int CARVEOUT_SMALL_KB = 64;    // sweep (2 KB a CTA), corrector, verification
 constexpr int CARVEOUT_GEMM_KB = 132;    // a dense-product CTA (up to 97 KB) beside six sweep CTAs
 
-template <typename Kernel>
-inline cudaError_t prefer_carveout(Kernel kernel, int kb) {
-  static std::atomic<unsigned long long> done{0};
+// Sets the carveout preference of `func` on the current device once (kernels of the same
+// signature are distinct entries: the registry is keyed by the function's address).
+inline cudaError_t prefer_carveout_fn(const void* func, int kb) {
+  static std::mutex mu;
+  static std::vector<std::pair<const void*, int>> done;
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
-  const unsigned long long bit = 1ull << (dev & 63);
-  if (done.load(std::memory_order_relaxed) & bit) return cudaSuccess;
+  std::lock_guard<std::mutex> lock(mu);
+  for (const auto& d : done)
+    if (d.first == func && d.second == dev) return cudaSuccess;
   int max_smem = 0;
   e = cudaDeviceGetAttribute(&max_smem, cudaDevAttrMaxSharedMemoryPerMultiprocessor, dev);
   if (e != cudaSuccess) return e;
   int pct = max_smem > 0 ? (kb * 1024 * 100 + max_smem - 1) / max_smem : 100;
   if (pct > 100) pct = 100;
-  e = cudaFuncSetAttribute(kernel, cudaFuncAttributePreferredSharedMemoryCarveout, pct);
-  if (e == cudaSuccess) done.fetch_or(bit, std::memory_order_relaxed);
+  e = cudaFuncSetAttribute(func, cudaFuncAttributePreferredSharedMemoryCarveout, pct);
+  if (e == cudaSuccess) done.emplace_back(func, dev);
   return e;
+}
+
+template <typename Kernel>
+inline cudaError_t prefer_carveout(Kernel kernel, int kb) {
+  return prefer_carveout_fn(reinterpret_cast<const void*>(kernel), kb);
 }
 
 __device__ __forceinline__ void set_status(int32_t* status, int code) {

@@ -135,6 +135,17 @@ def test_unaligned_rows_and_base(brisk):
     _run_and_check(brisk, wl, weights, block)
 
 
+def test_overlap_schedule_matches_unfused(brisk):
+    """At least 2432 rows (one proposal-sweep task per row) take the overlapping schedule: the
+    verifier sweep from the start, 256-wide tiles for the hidden projection. Bit for bit the
+    same as the three separate calls (narrow tiles, serial), and parity with the oracle."""
+    wl = synth.Workload("overlap", B=80, L=32, V=4096, d=512, K=8, r=256)
+    weights = _to(synth.make_weights(wl, "cpu"), "cuda")
+    block = _to(synth.make_block(wl, "cpu"), "cuda")
+    rep, g = _run_and_check(brisk, wl, weights, block, seqs=[0, 1, 40, 79], unfused=True)
+    assert rep.sequences == 4
+
+
 def test_non_finite_row_sets_numeric_status(brisk):
     wl = synth.Workload("nan", B=1, L=3, V=512, d=16, K=4, r=16)
     weights = _to(synth.make_weights(wl, "cpu"), "cuda")
