@@ -47,3 +47,34 @@ def test_graph_replays_match_direct_calls(brisk, kw):
         assert torch.equal(g.anchor, direct[s]["next_anchor"])
     g.close()
     assert tail.device_status() == brisk.OK
+
+
+def test_double_buffered_graph_loop_matches_direct_calls(brisk):
+    """Two captured graphs over two input buffer sets, the next block copied in on a second
+    stream while the current one runs, the anchor chained on the device: the same results as
+    direct calls on the same sequence of blocks."""
+    import bench
+    wl = synth.Workload("graphloop", B=2, L=8, V=4099, d=64, K=8, r=32, agree0=0.9,
+                        agree_decay=0.97, weight_std=0.2)
+    w = synth.make_weights(wl, "cuda")
+    pool = [synth.make_block(wl, "cuda", block=j) for j in range(3)]
+    tail = brisk.DecodeTail.for_workload(wl, w)
+    tail.prepare()
+    sm, vm = brisk.mode_ids(wl.select_mode, wl.verify_mode)
+    blocks = 7
+    direct = []
+    x0 = pool[0]["x0"].clone()
+    for t in range(blocks):
+        out = tail.tail(pool[t % len(pool)], sm, vm, x0=x0)
+        torch.cuda.synchronize()
+        direct.append({k: v.clone() for k, v in out.items()})
+        x0 = out["next_anchor"].clone()
+    stream = torch.cuda.Stream()
+    ms, nbytes, outs = bench.graph_loop_double_buffered(tail, pool, sm, vm, stream, blocks,
+                                                        keep=True)
+    assert ms > 0 and nbytes > 0 and len(outs) == blocks
+    for t in range(blocks):
+        for k in ("accepted_len", "out_tokens", "correction", "sel_tokens", "refined",
+                  "cand_ids", "next_anchor"):
+            assert torch.equal(outs[t][k], direct[t][k]), (t, k)
+    assert tail.device_status() == brisk.OK
