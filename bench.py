@@ -80,6 +80,13 @@ def sweep_source_hash() -> str:
     return hashlib.sha1(code.encode()).hexdigest()[:12]
 
 
+def workload_config(wl) -> dict:
+    """The workload keys of the bench line's config (the same in both arms)."""
+    return {"workload": WORKLOAD, "B": wl.B, "L": wl.L, "V": wl.V, "d": wl.d, "K": wl.K,
+            "r": wl.r, "input_dtype": "bf16", "select": wl.select_mode,
+            "verify": wl.verify_mode, "parallelism": "replicas"}
+
+
 def sweep_span_ms(q0, q1, p0, p1) -> float:
     """Milliseconds from the earlier of the two sweep launches' start events to the later of
     their end events (all offsets taken from q0, so either launch may start first)."""
@@ -292,8 +299,8 @@ def run_reference(args):
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000.0 * tot_s / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic",
-        "config": {"workload": WORKLOAD, "B": 1, "L": wl.L, "V": wl.V, "d": wl.d, "K": wl.K,
-                   "r": wl.r, "step": "one sequence of one block per step"},
+        "config": {**workload_config(wl),
+                   "sample": "each step times the oracle on one sequence of one block"},
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
                          "sample": "one sequence of the decode-stream workload per step"},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
@@ -463,9 +470,7 @@ def run_ours(args):
         "warmup": args.warmup, "ms_per_step": 1000.0 * elapsed_max / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
         "data": "synthetic",
-        "config": {"workload": WORKLOAD, "B": wl.B, "L": wl.L, "V": wl.V, "d": wl.d, "K": wl.K,
-                   "r": wl.r, "input_dtype": "bf16", "select": wl.select_mode,
-                   "verify": wl.verify_mode, "parallelism": "replicas",
+        "config": {**workload_config(wl),
                    "l2": f"inputs larger than L2 ({sweep_bytes / 1e9:.2f} GB of logits per step,"
                          f" {pool_n} distinct blocks cycled)",
                    "prepare_ms": round(prepare_ms, 1)},
