@@ -16,10 +16,15 @@ Language Models"):
   rejection rate at position i among the blocks whose verification reached i.
 * Sec. 3.2, Eq. 3 (risk-reward weights): w_i^raw = -dFPT/dz_i = -dFPT/da_i * a_i (1 - a_i) with
   z_i = log(a_i / (1 - a_i)); w_bar_i = M w_i^raw / (sum_j w_j^raw + eps).
+* App. C.1, Eq. 8 (the instantiation for ISD verification, which the paper uses for
+  its FPT and weights): TPF(a) = (2 + sum_{k=1}^{M-1} A_k) / (2 - A_M) with M = N - 1; the same
+  as Eq. 2 with gains g_k = 2 + min(k, M - 1) and costs c_k = 2 (k < M), c_M = 1.
 
 Positions are 0-based here (position i of the paper is index i-1); A has M+1 entries with
 A[0] = 1. Parity pins: the paper's printed TPF_8 values, the unit-cost identity, the length
-law summing to one, E[L] = sum A_k, the weights against finite differences of FPT.
+law summing to one, E[L] = sum A_k, the weights against finite differences of FPT, Eq. 8
+against Eq. 2 with its stated costs and, at a constant profile, against the Sec. 2.2 rule and
+the printed TPF_8 values.
 """
 from __future__ import annotations
 
@@ -78,6 +83,21 @@ def fpt(a, g, c):
 def unit_costs(M: int):
     """g_k = k + 1 committed tokens (the accepted prefix plus one), c_k = 1 forward pass."""
     return np.arange(M + 1, dtype=np.float64) + 1.0, np.ones(M + 1)
+
+
+def isd_costs(M: int):
+    """Eq. 8's gains and costs for Eq. 2: g_k = 2 + min(k, M - 1); c_k = 2 for k < M, c_M = 1."""
+    g = np.array([2.0 + min(k, M - 1) for k in range(M + 1)])
+    c = np.array([2.0] * M + [1.0])
+    return g, c
+
+
+def tpf_isd_profile(a) -> float:
+    """Eq. 8: TPF(a) = (2 + sum_{k=1}^{M-1} A_k) / (2 - A_M) for a profile of M positions."""
+    a = np.asarray(a, dtype=np.float64)
+    M = len(a)
+    A = survival(a)
+    return float((2.0 + sum(A[k] for k in range(1, M))) / (2.0 - A[M]))
 
 
 def tpf_isd(N: int, r: float) -> float:

@@ -100,3 +100,41 @@ def test_profile_recovers_a_known_law_statistically():
     a = A.profile(reach, accept)
     se = np.sqrt(a_true * (1 - a_true) / reach)
     assert np.all(np.abs(a - a_true) < 5 * se)
+
+
+def test_isd_instantiation_equals_renewal_reward_with_its_costs():
+    """Eq. 8's closed form against Eq. 2 evaluated with the gains and costs the paper states for
+    it (two independent formulas)."""
+    rng = np.random.default_rng(5)
+    for M in (1, 2, 3, 7, 15, 31):
+        for _ in range(5):
+            a = rng.uniform(0.0, 1.0, M)
+            g, c = A.isd_costs(M)
+            assert abs(A.tpf(a, g, c) - A.tpf_isd_profile(a)) < 1e-12 * A.tpf_isd_profile(a)
+
+
+@pytest.mark.parametrize("N,r,t", _golden())
+def test_isd_instantiation_at_constant_profile_gives_printed_values(N, r, t):
+    """At a_i = 1 - r (M = N - 1 positions) Eq. 8 is the Sec. 2.2 rule: the printed TPF_8."""
+    a = np.full(N - 1, 1.0 - r)
+    assert abs(A.tpf_isd_profile(a) - A.tpf_isd(N, r)) < 1e-12
+    assert abs(A.tpf_isd_profile(a) - t) <= 0.005
+
+
+def test_isd_weights_match_finite_differences():
+    rng = np.random.default_rng(6)
+    M = 7
+    a = rng.uniform(0.3, 0.97, M)
+    g, c = A.isd_costs(M)
+    w_raw, w_bar = A.weights(a, g, c)
+    z = np.log(a / (1 - a))
+    h = 1e-6
+    for i in range(M):
+        zp, zm = z.copy(), z.copy()
+        zp[i] += h
+        zm[i] -= h
+        fp = 1.0 / A.tpf_isd_profile(1 / (1 + np.exp(-zp)))
+        fm = 1.0 / A.tpf_isd_profile(1 / (1 + np.exp(-zm)))
+        fd = -(fp - fm) / (2 * h)
+        assert abs(fd - w_raw[i]) < 1e-7 * max(1.0, abs(fd))
+    assert abs(w_bar.mean() - 1.0) < 1e-6
