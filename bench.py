@@ -392,6 +392,8 @@ def run_ours(args):
     reach_h, accept_h = counts_h[:wl.L], counts_h[wl.L:]
     prof_a = [accept_h[i] / reach_h[i] if reach_h[i] else 0.0 for i in range(wl.L)]
     prof_tpf, _, prof_w = brisk.acceptance_weights(prof_a)
+    # the ISD instantiation (App. C.1, Eq. 8), which the paper uses for FPT and the weights
+    isd_tpf, _, isd_w = brisk.acceptance_weights(prof_a, *brisk.isd_costs(wl.L))
     # distillation loss of the head (App. C.3) on one block's outputs: kernel time, untimed above
     full = tail.alloc_outputs(full=True)
     tail.tail(pool[0], sm, vm, out=full)
@@ -493,7 +495,9 @@ def run_ours(args):
         "acceptance_profile": {"a": [round(x, 4) for x in prof_a[:8]],
                                "positions_shown": min(8, wl.L),
                                "tpf_unit_cost": prof_tpf,
-                               "w_bar": [round(x, 4) for x in prof_w[:8]]},
+                               "w_bar": [round(x, 4) for x in prof_w[:8]],
+                               "tpf_isd_eq8": isd_tpf,
+                               "w_bar_isd_eq8": [round(x, 4) for x in isd_w[:8]]},
         "graph_loop": graph_loop,
         "distill_loss_us": distill_us,
         "replay": {"first_breakers": n_fb,

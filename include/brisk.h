@@ -315,6 +315,13 @@ brisk_status brisk_distill_loss(const brisk_dims *dims, const void *logits_p,
                                 const float *refined, const int32_t *accepted_len, float beta,
                                 float *loss, float *grad_refined, void *workspace, void *stream);
 
+/* Host-side: the gains and costs that make Eq. 2 the ISD instantiation the paper uses for FPT
+ * and the weights (App. C.1, Eq. 8: TPF = (2 + sum_{k=1}^{M-1} A_k) / (2 - A_M), M = N - 1):
+ * g[k] = 2 + min(k, M - 1) and c[k] = 2 for k < M, c[M] = 1, written for k = 0..M (M + 1 values
+ * each, caller-owned host arrays), to pass to brisk_acceptance_weights. BRISK_ERR_INVALID_ARG
+ * for M outside 1..64 or a NULL array. */
+brisk_status brisk_isd_costs(int32_t M, double *g, double *c);
+
 /* Host-side: tokens per forward of the ISD stride-N rule at constant rejection r (Sec. 2.2):
  * (2 + sum_{i=1}^{N-2} (1-r)^i) / (2 - (1-r)^{N-1}); NaN for N < 2 or r outside [0, 1]. */
 double brisk_tpf_isd(int32_t N, double r);

@@ -80,6 +80,7 @@ _SIGS = [
     ("brisk_acceptance_weights", ctypes.c_int,
      [ctypes.c_int32, _vp, _vp, _vp, ctypes.c_double, _vp, _vp, _vp]),
     ("brisk_tpf_isd", ctypes.c_double, [ctypes.c_int32, ctypes.c_double]),
+    ("brisk_isd_costs", ctypes.c_int, [ctypes.c_int32, ctypes.c_void_p, ctypes.c_void_p]),
     ("brisk_tail_graph_create", ctypes.c_int,
      [ctypes.POINTER(Dims), ctypes.POINTER(Params), _vp, ctypes.POINTER(TailIO), ctypes.c_int32,
       ctypes.c_int32, _vp, _vp, ctypes.POINTER(_vp)]),
@@ -377,6 +378,16 @@ def acceptance_weights(a, g=None, c=None, eps: float = 1e-8):
     _check(lib().brisk_acceptance_weights(M, vp(a), vp(gg), vp(cc), float(eps), ctypes.byref(tpf),
                                           vp(w_raw), vp(w_bar)), "acceptance_weights")
     return tpf.value, w_raw, w_bar
+
+
+def isd_costs(M: int):
+    """Gains g[0..M] and costs c[0..M] of the ISD instantiation (App. C.1, Eq. 8)."""
+    import numpy as np
+    g = np.zeros(int(M) + 1, dtype=np.float64)
+    c = np.zeros(int(M) + 1, dtype=np.float64)
+    _check(lib().brisk_isd_costs(int(M), g.ctypes.data_as(ctypes.c_void_p),
+                                 c.ctypes.data_as(ctypes.c_void_p)), "isd_costs")
+    return g, c
 
 
 def tpf_isd(N: int, r: float) -> float:

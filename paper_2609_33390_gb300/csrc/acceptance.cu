@@ -63,6 +63,15 @@ extern "C" double brisk_tpf_isd(int32_t N, double r) {
   return num / (2.0 - qi * q);   // qi * q = q^(N-1)
 }
 
+extern "C" brisk_status brisk_isd_costs(int32_t M, double* g, double* c) {
+  if (M < 1 || M > 64 || !g || !c) return BRISK_ERR_INVALID_ARG;
+  for (int k = 0; k <= M; ++k) {
+    g[k] = 2.0 + (k < M - 1 ? k : M - 1);
+    c[k] = k < M ? 2.0 : 1.0;
+  }
+  return BRISK_OK;
+}
+
 extern "C" brisk_status brisk_acceptance_weights(int32_t M, const double* a, const double* g,
                                                  const double* c, double eps, double* tpf,
                                                  double* w_raw, double* w_bar) {

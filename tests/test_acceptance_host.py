@@ -57,3 +57,19 @@ def test_invalid_profiles_rejected(B):
         B.acceptance_weights(np.array([np.nan]))
     with pytest.raises(B.BriskError):
         B.acceptance_weights(np.full(65, 0.5))
+
+
+@pytest.mark.parametrize("M", [1, 2, 7, 64])
+def test_isd_costs_and_weights_match_oracle(B, M):
+    g, c = B.isd_costs(M)
+    og, oc = A.isd_costs(M)
+    np.testing.assert_array_equal(g, og)
+    np.testing.assert_array_equal(c, oc)
+    a = np.random.default_rng(10 + M).uniform(0.2, 0.99, M)
+    tpf, w_raw, w_bar = B.acceptance_weights(a, g, c, eps=1e-8)
+    assert abs(tpf - A.tpf_isd_profile(a)) <= 1e-12 * tpf
+    ow_raw, ow_bar = A.weights(a, og, oc, eps=1e-8)
+    np.testing.assert_allclose(w_raw, ow_raw, rtol=1e-10, atol=1e-15)
+    np.testing.assert_allclose(w_bar, ow_bar, rtol=1e-10, atol=1e-15)
+    with pytest.raises(B.BriskError):
+        B.isd_costs(0)
