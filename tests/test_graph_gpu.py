@@ -18,7 +18,9 @@ def brisk():
 
 @pytest.mark.parametrize("kw", [dict(B=2, L=8, V=4099, d=64, K=8, r=32),
                                 dict(B=3, L=12, V=5003, d=64, K=4, r=16, select_mode="sample",
-                                     verify_mode="stochastic")])
+                                     verify_mode="stochastic"),
+                                # 2560 rows: the overlapping schedule (three side streams)
+                                dict(B=80, L=32, V=4096, d=512, K=8, r=256)])
 def test_graph_replays_match_direct_calls(brisk, kw):
     wl = synth.Workload("graph", agree0=0.9, agree_decay=0.97, weight_std=0.2, **kw)
     w = synth.make_weights(wl, "cuda")
