@@ -513,62 +513,6 @@ def run_ours(args):
     return 0
 
 
-BLOCK_INPUTS = ("logits_q", "logits_p", "hidden", "h_c", "u_sel", "u_acc", "u_res")
-
-
-def graph_loop_double_buffered(tail, pool, sm, vm, stream, blocks, keep=False):
-    """Block after block through two captured decode tails (App. F), one per input buffer set,
-    the anchor chained on the device through one buffer both graphs share. While block t runs
-    on `stream`, a second stream copies block t+1's inputs from `pool` (pre-generated blocks,
-    taken in turn) into the other buffer set: the stand-in for the backbone writing the next
-    block. Events order the two streams: block t waits for its set to be filled, the refill of
-    a set waits for the block that last read it.
-
-    Returns (elapsed ms of the `blocks` replays on `stream`, bytes copied per block, per-block
-    output copies if keep else None)."""
-    import torch
-    anchor = pool[0]["x0"].clone()
-    bufs = []
-    for j in range(2):
-        b = {k: pool[j % len(pool)][k].clone() for k in BLOCK_INPUTS}
-        b["x0"] = anchor
-        bufs.append(b)
-    out = tail.alloc_outputs(full=keep)
-    out["next_anchor"] = anchor
-    torch.cuda.synchronize()
-    graphs = [tail.graph(bufs[j], sm, vm, out=out, chain_anchor=False, stream=stream)
-              for j in range(2)]
-    prod = torch.cuda.Stream()
-    ready = [torch.cuda.Event(), torch.cuda.Event()]
-    done = [torch.cuda.Event(), torch.cuda.Event()]
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    nbytes = sum(bufs[0][k].numel() * bufs[0][k].element_size() for k in BLOCK_INPUTS)
-    outs = [] if keep else None
-    ready[0].record(prod)
-    e0.record(stream)
-    for t in range(blocks):
-        k, nk = t % 2, 1 - t % 2
-        with torch.cuda.stream(prod):
-            if t >= 1:
-                prod.wait_event(done[nk])
-            src = pool[(t + 1) % len(pool)]
-            for name in BLOCK_INPUTS:
-                bufs[nk][name].copy_(src[name], non_blocking=True)
-            ready[nk].record(prod)
-        stream.wait_event(ready[k])
-        graphs[k].launch()
-        done[k].record(stream)
-        if keep:
-            with torch.cuda.stream(stream):
-                outs.append({n: v.clone() for n, v in out.items()})
-    e1.record(stream)
-    stream.synchronize()
-    prod.synchronize()
-    for g in graphs:
-        g.close()
-    return e0.elapsed_time(e1), nbytes, outs
-
-
 def run_graph_loop(dev, blocks=30):
     """Per-block latency of the decode tail on one sequence (the `single` workload), as direct
     calls and as replays of the captured CUDA graph (App. F), anchors chained on the device."""
@@ -608,6 +552,7 @@ def run_graph_loop(dev, blocks=30):
     g.close()
     # new inputs every block: double-buffered graphs, the next block copied in on a second stream
     pool = [synth.make_block(wl, dev, block=j) for j in range(4)]
+    from paper_2609_33390_gb300.loop import graph_loop_double_buffered
     graph_loop_double_buffered(tail, pool, sm, vm, stream, 5)
     ms, nbytes, _ = graph_loop_double_buffered(tail, pool, sm, vm, stream, blocks)
     return {"workload": "single", "B": wl.B, "L": wl.L, "V": wl.V, "blocks": blocks,

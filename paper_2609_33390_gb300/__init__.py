@@ -1,12 +1,13 @@
 """BRISK-DLM decode tail on GB300 (sm_103a).
 
 The compute runs in the CUDA library built from ``csrc/``; ``brisk`` is its
-thin ctypes binding (loaded on first use). ``synth`` builds seeded synthetic
-inputs shaped like the paper's workloads.
+thin ctypes binding (loaded on first use); ``loop`` drives captured tails block after
+block with double-buffered inputs. ``synth`` builds seeded synthetic inputs shaped like the
+paper's workloads.
 """
 import importlib
 
-__all__ = ["synth", "brisk", "build"]
+__all__ = ["synth", "brisk", "build", "loop"]
 
 
 def __getattr__(name):

@@ -55,7 +55,7 @@ def test_double_buffered_graph_loop_matches_direct_calls(brisk):
     """Two captured graphs over two input buffer sets, the next block copied in on a second
     stream while the current one runs, the anchor chained on the device: the same results as
     direct calls on the same sequence of blocks."""
-    import bench
+    from paper_2609_33390_gb300.loop import graph_loop_double_buffered
     wl = synth.Workload("graphloop", B=2, L=8, V=4099, d=64, K=8, r=32, agree0=0.9,
                         agree_decay=0.97, weight_std=0.2)
     w = synth.make_weights(wl, "cuda")
@@ -72,8 +72,7 @@ def test_double_buffered_graph_loop_matches_direct_calls(brisk):
         direct.append({k: v.clone() for k, v in out.items()})
         x0 = out["next_anchor"].clone()
     stream = torch.cuda.Stream()
-    ms, nbytes, outs = bench.graph_loop_double_buffered(tail, pool, sm, vm, stream, blocks,
-                                                        keep=True)
+    ms, nbytes, outs = graph_loop_double_buffered(tail, pool, sm, vm, stream, blocks, keep=True)
     assert ms > 0 and nbytes > 0 and len(outs) == blocks
     for t in range(blocks):
         for k in ("accepted_len", "out_tokens", "correction", "sel_tokens", "refined",
