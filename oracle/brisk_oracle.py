@@ -316,14 +316,21 @@ class VerifyResult:
     accept_margins: Optional[np.ndarray] = None  # [L] |u_acc - alpha| per decided position
 
 
-def residual_sample(row_p: np.ndarray, pi_ids: Sequence[int], pi_mass: Sequence[float], u: float):
-    """Draw from the normalised positive part [p - pi]_+ with one uniform u, walking ids
-    in ascending order; Z <= Z_FLOOR falls back to argmax p. Returns (id, margin)."""
+def residual_mass(row_p: np.ndarray, pi_ids: Sequence[int], pi_mass: Sequence[float]) -> np.ndarray:
+    """The unnormalised residual R(v) = max(0, p(v) - pi(v)) over the whole vocabulary
+    (Sec. 3.3, speculative sampling), with pi(v) = 0 outside the candidate ids."""
     lse = log_partition(row_p)
     p = np.exp(np.asarray(row_p, dtype=np.float64) - lse)
     R = p.copy()
     for v, m in zip(pi_ids, pi_mass):
         R[int(v)] = max(0.0, p[int(v)] - float(m))
+    return R
+
+
+def residual_sample(row_p: np.ndarray, pi_ids: Sequence[int], pi_mass: Sequence[float], u: float):
+    """Draw from the normalised positive part [p - pi]_+ with one uniform u, walking ids
+    in ascending order; Z <= Z_FLOOR falls back to argmax p. Returns (id, margin)."""
+    R = residual_mass(row_p, pi_ids, pi_mass)
     Z = R.sum()
     if Z <= Z_FLOOR:
         return verifier_argmax(row_p), np.inf
@@ -376,6 +383,14 @@ def verify_sequence(rows_p: Callable[[int], np.ndarray], sel_tokens: np.ndarray,
         out[i] = corr
         return VerifyResult(i, out, int(corr), acc_margin, res_margin, margins)
     return VerifyResult(L, out, -1, acc_margin, np.inf, margins)
+
+
+def next_anchor(vr: VerifyResult, sel_tokens: Sequence[int]) -> int:
+    """The anchor of the next block (Algorithm 1(b), commit step): the last token this block
+    commits, which is the correction at the first rejection, or the last selected token when
+    the whole block is accepted (no bonus token is drawn, see the verification readings)."""
+    L = len(sel_tokens)
+    return int(vr.correction) if vr.accepted_len < L else int(sel_tokens[L - 1])
 
 
 # ---------------------------------------------------------------------------

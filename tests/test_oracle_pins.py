@@ -453,3 +453,64 @@ def test_mean_accepted_prefix_follows_survival_law():
     expect = np.cumprod(acc).sum()
     se = lens.std() / math.sqrt(n)
     assert abs(lens.mean() - expect) < 4.5 * se, (lens.mean(), expect, se)
+
+
+# ---------------------------------------------------------------------------
+# Commit step (Algorithm 1(b)): the anchor of the next block
+# ---------------------------------------------------------------------------
+
+def test_next_anchor_is_the_last_committed_token():
+    """The next block's anchor is the last token this block commits: the correction when a
+    position is rejected, the last selection when the whole block is accepted. Checked against
+    the out_tokens row read independently (its last entry >= 0) over random stochastic blocks
+    whose rejections fall at every position."""
+    L, V, K = 6, 12, 4
+    rng = np.random.default_rng(77)
+    seen = set()
+    for _ in range(300):
+        lq = rng.normal(size=(L, V)) * 2.0
+        lpv = lq + rng.normal(size=(L, V)) * rng.uniform(0.0, 3.0)
+        cand = np.array([O.ranked_ids(lq[i])[:K] for i in range(L)])
+        refined = np.array([lq[i][cand[i]] for i in range(L)]) + rng.normal(size=(L, K))
+        ranks = rng.integers(0, K, size=L)
+        sel = cand[np.arange(L), ranks]
+        vr = O.verify_sequence(lambda i: lpv[i], sel, cand, refined, O.SAMPLE, O.STOCHASTIC,
+                               rng.uniform(size=L), rng.uniform(size=L))
+        committed = [int(t) for t in vr.out_tokens if t >= 0]
+        assert len(committed) == min(vr.accepted_len + 1, L)
+        assert O.next_anchor(vr, sel) == committed[-1]
+        seen.add(vr.accepted_len)
+    assert seen == set(range(L + 1))   # every rejection position and the full block
+
+
+def test_next_anchor_closed_cases():
+    L, V, K = 5, 30, 4
+    lq = RNG.normal(size=(L, V))
+    cand = np.array([O.ranked_ids(lq[i])[:K] for i in range(L)])
+    sel = cand[:, 0]
+    # identical distributions, greedy, the base ranking: the whole block, anchor = last token
+    vr = O.verify_sequence(lambda i: lq[i], sel, cand, np.zeros((L, K)))
+    assert vr.accepted_len == L and O.next_anchor(vr, sel) == sel[-1]
+    # the verifier's argmax at position 0 outside the candidates: anchor = that argmax
+    lpv = lq.copy()
+    outside = [v for v in range(V) if v not in cand[0]][0]
+    lpv[0, outside] = 50.0
+    vr = O.verify_sequence(lambda i: lpv[i], sel, cand, np.zeros((L, K)))
+    assert vr.accepted_len == 0 and O.next_anchor(vr, sel) == outside
+
+
+def test_residual_mass_is_one_minus_the_acceptance_rate():
+    """sum_v [p(v) - pi(v)]_+ = 1 - sum_v min(p(v), pi(v)) for a proposal law pi on the
+    candidates: the residual's mass is the rejection probability (Sec. 3.3)."""
+    rng = np.random.default_rng(5)
+    for _ in range(50):
+        V, K = 40, 6
+        row = rng.normal(size=V) * 2
+        p = scipy.special.softmax(row)
+        ids = rng.choice(V, size=K, replace=False)
+        pi = scipy.special.softmax(rng.normal(size=K))
+        R = O.residual_mass(row, ids, pi)
+        assert np.all(R >= 0)
+        pim = np.zeros(V)
+        pim[ids] = pi
+        assert abs(R.sum() - (1.0 - np.minimum(p, pim).sum())) < 1e-12
