@@ -60,14 +60,26 @@ class Report:
     notes: list = field(default_factory=list)
 
 
+def residual_neighbours(row_p: np.ndarray, pi_ids, pi_mass, v: int):
+    """The ids on either side of v with positive residual [p - pi]_+ (the only other outcomes
+    an inverse-CDF draw that lands near one of v's boundaries can give); None where none."""
+    R = O.residual_mass(row_p, pi_ids, pi_mass)
+    pos = np.nonzero(R > 0)[0]
+    below = pos[pos < v]
+    above = pos[pos > v]
+    return (int(below[-1]) if below.size else None, int(above[0]) if above.size else None)
+
+
 def check_sequence(b: int, block: dict, params: O.Params, K: int, gpu: dict, select_mode: str,
-                   verify_mode: str, rep: Report) -> None:
-    """Compare sequence b of the GPU outputs `gpu` (numpy) with the oracle."""
+                   verify_mode: str, rep: Report, x0=None):
+    """Compare sequence b of the GPU outputs `gpu` (numpy) with the oracle; x0 overrides the
+    block's anchor (a chained block starts from the previous block's last committed token).
+    Returns the oracle's (corrector trace, verify result) of the accepted run."""
     lq = np64(block["logits_q"][b])
     lpv = np64(block["logits_p"][b])
     hidden = np64(block["hidden"][b])
     h_c = np64(block["h_c"][b])
-    x0 = int(block["x0"][b])
+    x0 = int(block["x0"][b]) if x0 is None else int(x0)
     L = lq.shape[0]
     u_sel = block["u_sel"][b].cpu().numpy().astype(np.float64)
     u_acc = block["u_acc"][b].cpu().numpy().astype(np.float64)
@@ -116,6 +128,12 @@ def check_sequence(b: int, block: dict, params: O.Params, K: int, gpu: dict, sel
         gc = int(gpu["correction"][b])
         if gc != vr.correction and verify_mode == O.STOCHASTIC and force_corr is None \
                 and vr.resample_margin < TIE_TOL:
+            # only the neighbouring id with residual mass across the boundary is also correct
+            j = vr.accepted_len
+            rank = int(np.nonzero(cand[j] == tr.sel_tokens[j])[0][0])
+            pi = O.proposal_law(tr.refined[j], select_mode, rank)
+            assert gc in residual_neighbours(lpv[j], cand[j], pi, vr.correction), \
+                f"correction seq {b}: gpu {gc} is not a neighbour of the oracle's {vr.correction}"
             force_corr = gc
             rep.near_ties += 1
             rep.notes.append(f"seq {b}: residual near-tie")
@@ -123,8 +141,12 @@ def check_sequence(b: int, block: dict, params: O.Params, K: int, gpu: dict, sel
         assert gc == vr.correction, f"correction seq {b}: gpu {gc} oracle {vr.correction}"
         np.testing.assert_array_equal(gpu["out_tokens"][b], vr.out_tokens,
                                       err_msg=f"out_tokens seq {b}")
+        if "next_anchor" in gpu:
+            na = O.next_anchor(vr, tr.sel_tokens)
+            assert int(gpu["next_anchor"][b]) == na, \
+                f"next_anchor seq {b}: gpu {int(gpu['next_anchor'][b])} oracle {na}"
         rep.sequences += 1
-        return
+        return tr, vr
     raise AssertionError(f"seq {b}: too many near-tie re-runs")
 
 

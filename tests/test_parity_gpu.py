@@ -224,6 +224,16 @@ def test_workload_parity_full_size(brisk, name):
     rep, g = _run_and_check(brisk, wl, weights, block, seqs=seqs, unfused=(name == "single"))
     assert rep.sequences == len(seqs)
     assert rep.near_ties <= max(1, len(seqs) * wl.L // 50), rep.notes
+    # step 1 of every row against the oracle (the rows of the sequences not checked above too)
+    if B > 16:
+        import oracle_pool
+        BL = B * wl.L
+        rows = block["logits_q"].float().reshape(BL, wl.V).cpu().numpy()
+        ids, lp, lse = oracle_pool.topk_all_rows(rows, wl.K)
+        np.testing.assert_array_equal(g["cand_ids"].reshape(BL, wl.K), ids)
+        e = np.abs(g["cand_logprob"].reshape(BL, wl.K) - lp)
+        assert np.where(np.isfinite(lp), e, 0.0).max() <= 1e-3
+        assert np.abs(g["lse_q"].reshape(BL) - lse).max() <= 1e-3
     # every sequence's invariants, checked or not
     a = g["accepted_len"]
     assert np.all((a >= 0) & (a <= wl.L))

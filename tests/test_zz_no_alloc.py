@@ -2,13 +2,15 @@
 (a plug-in handed only its input and output buffers, an engine whose memory manager owns all of
 HBM, a decode loop that must not allocate). It must agree with brisk_topk_candidates, which
 uses a caller workspace, on two calls in a row: the second call reuses the library's fixed
-scratch array that the first call left behind."""
+scratch array that the first call left behind. Both calls are also checked against the oracle's
+candidates row by row."""
 import ctypes
 
 import numpy as np
 import pytest
 import torch
 
+from oracle import brisk_oracle as O
 from paper_2609_33390_gb300 import synth
 
 ATOL = 1e-3
@@ -57,3 +59,12 @@ def test_noalloc_matches_workspace_entry_point_twice(B):
                                    atol=ATOL, err_msg=f"call {call}")
         np.testing.assert_allclose(lse.cpu().numpy(), ref["lse_q"].cpu().numpy(), rtol=0,
                                    atol=ATOL, err_msg=f"call {call}")
+        # and against the oracle's candidates, row by row
+        rows = lq.float().reshape(-1, wl.V).cpu().numpy().astype(np.float64)
+        ids_h = ids.reshape(-1, wl.K).cpu().numpy()
+        lp_h = lp.reshape(-1, wl.K).cpu().numpy()
+        lse_h = lse.reshape(-1).cpu().numpy()
+        for j in range(rows.shape[0]):
+            o_ids, o_lp, o_lse = O.topk_candidates(rows[j], wl.K)
+            np.testing.assert_array_equal(ids_h[j], o_ids, err_msg=f"call {call} row {j}")
+            assert np.abs(lp_h[j] - o_lp).max() <= ATOL and abs(lse_h[j] - o_lse) <= ATOL
