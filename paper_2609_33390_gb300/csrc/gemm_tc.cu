@@ -7,8 +7,9 @@
 // tcgen05.commit. The epilogue reads TMEM 32 columns at a time (tcgen05.ld), stages each chunk
 // in one of several shared-memory buffers (the ring is free by then) and writes it with a TMA
 // tensor store, so that staging the next chunks overlaps the stores in flight. Every wait on
-// an mbarrier is bounded (about 2 s of SM clock): on expiry the CTA records BRISK_ERR_TIMEOUT,
-// drains what it started and frees its TMEM.
+// an mbarrier is bounded (a kernel argument, by default about 2 s of SM clock): on expiry the
+// CTA records BRISK_ERR_TIMEOUT, drains what it started (its TMA loads and the tensor-core
+// operations it issued, each drain wait bounded by the default limit) and frees its TMEM.
 //
 // Used for the corrector's one dense contraction (the MASK hidden states times
 // the hidden projection, App. C.3 "64-dimensional projection of the MASK
@@ -28,7 +29,8 @@ constexpr int TC_BM = 128;
 constexpr int TC_BK = 64;               // one 128-byte swizzle row of bf16
 constexpr int TC_STAGES_MAX = 4;
 constexpr int TC_THREADS = 128;
-constexpr long long WAIT_LIMIT_CYCLES = 4000000000ll;   // about 2 s of SM clock per wait
+constexpr long long DRAIN_LIMIT_CYCLES = 4000000000ll;  // about 2 s of SM clock per drain wait
+constexpr long long SHORT_WAIT_CYCLES = 1ll << 20;      // below this, waits poll without suspending
 
 __device__ __forceinline__ uint32_t su32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -52,14 +54,43 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
       : "memory");
   return ok != 0;
 }
-// Bounded wait for the phase with the given parity; false on expiry or abort. The SM cycle
-// counter and the abort flag are only read every 64 polls.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag) {
+// Non-blocking test of the phase with the given parity (never suspends the thread).
+__device__ __forceinline__ bool mbar_test(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(su32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+// Bounded wait for the phase with the given parity; false on expiry (more than `limit` SM
+// cycles) or abort. With a long limit the thread may suspend in try_wait and the cycle counter
+// and the abort flag are read every 64 polls; a short limit (tests of the failure path) polls
+// with test_wait and reads the counter every poll, so that it expires after `limit` cycles.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
+                                          long long limit) {
+  if (limit < SHORT_WAIT_CYCLES) {
+    const long long t0 = clock64();
+    for (;;) {
+      if (mbar_test(bar, parity)) return true;
+      if (*abort_flag || clock64() - t0 > limit) return false;
+    }
+  }
   if (mbar_try_wait(bar, parity)) return true;
   const long long t0 = clock64();
   for (unsigned n = 1;; ++n) {
     if (mbar_try_wait(bar, parity)) return true;
-    if ((n & 63) == 0 && (*abort_flag || clock64() - t0 > WAIT_LIMIT_CYCLES)) return false;
+    if ((n & 63) == 0 && (*abort_flag || clock64() - t0 > limit)) return false;
+  }
+}
+// Wait for a phase that is known to complete (the drain after an abort), bounded by the
+// default limit.
+__device__ __forceinline__ void mbar_drain(uint64_t* bar, uint32_t parity) {
+  const long long t0 = clock64();
+  while (!mbar_try_wait(bar, parity) && clock64() - t0 < DRAIN_LIMIT_CYCLES) {
   }
 }
 __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, uint64_t* bar, int x,
@@ -179,6 +210,7 @@ struct TcArgs {
   int tiles0;       // CTAs of problem 0
   int BN;           // tile columns (multiple of 16, <= 256), shared by both problems
   int tmem_cols;    // power of two >= max(32, BN)
+  long long wait_limit;   // SM cycles a pipeline or accumulator wait spins before it gives up
   int32_t* status;
 };
 
@@ -233,7 +265,8 @@ gemm_tc_kernel(const __grid_constant__ TcMaps maps, const __grid_constant__ TcAr
     // TMA producer
     for (int kb = 0; kb < nk; ++kb) {
       const int s = kb % TC_STAGES;
-      if (kb >= TC_STAGES && !mbar_wait(&empty[s], ((kb / TC_STAGES) & 1) ^ 1, abort_flag)) {
+      if (kb >= TC_STAGES &&
+          !mbar_wait(&empty[s], ((kb / TC_STAGES) & 1) ^ 1, abort_flag, a.wait_limit)) {
         *abort_flag = 1;
         break;
       }
@@ -247,7 +280,7 @@ gemm_tc_kernel(const __grid_constant__ TcMaps maps, const __grid_constant__ TcAr
     const uint32_t idesc = idesc_bf16(TC_BM, a.BN);
     for (int kb = 0; kb < nk; ++kb) {
       const int s = kb % TC_STAGES;
-      if (!mbar_wait(&full[s], (kb / TC_STAGES) & 1, abort_flag)) {
+      if (!mbar_wait(&full[s], (kb / TC_STAGES) & 1, abort_flag, a.wait_limit)) {
         *abort_flag = 1;
         break;
       }
@@ -262,25 +295,27 @@ gemm_tc_kernel(const __grid_constant__ TcMaps maps, const __grid_constant__ TcAr
     umma_commit(accum);
   }
   // epilogue: one thread waits for the accumulator (with back-off, so that polling does not
-  // compete with TMA and the MMAs for the shared-memory pipe); the others wait at the barrier
+  // compete with TMA and the MMAs for the shared-memory pipe); the others wait at the barrier.
+  // The MMA thread has issued its commit to `accum` before this barrier, aborted or not.
   __syncthreads();
   if (threadIdx.x == 0) {
     const long long t0 = clock64();
     bool done = false;
-    while (!(done = mbar_try_wait(accum, 0))) {
-      if (*abort_flag || clock64() - t0 > WAIT_LIMIT_CYCLES) break;
-      __nanosleep(128);
+    while (!(done = mbar_test(accum, 0))) {
+      if (*abort_flag || clock64() - t0 > a.wait_limit) break;
+      if (a.wait_limit >= SHORT_WAIT_CYCLES) __nanosleep(128);
     }
-    if (!done) *abort_flag = 1;
+    if (!done) {
+      *abort_flag = 1;
+      // the tensor-core operations already issued still write TMEM and read the ring: the
+      // commit covers all of them, so wait for it before TMEM is freed
+      mbar_drain(accum, 0);
+    }
   }
   // drain: the producer's loads complete on their own; wait (bounded) for the ones issued
   if (warp == 0 && lane == 0 && *abort_flag) {
-    for (int kb = (issued > TC_STAGES ? issued - TC_STAGES : 0); kb < issued; ++kb) {
-      const long long t0 = clock64();
-      while (!mbar_try_wait(&full[kb % TC_STAGES], (kb / TC_STAGES) & 1) &&
-             clock64() - t0 < WAIT_LIMIT_CYCLES) {
-      }
-    }
+    for (int kb = (issued > TC_STAGES ? issued - TC_STAGES : 0); kb < issued; ++kb)
+      mbar_drain(&full[kb % TC_STAGES], (kb / TC_STAGES) & 1);
   }
   __syncthreads();
   tc_fence_after();
@@ -401,6 +436,8 @@ bool make_out_map(CUtensorMap* map, const void* ptr, bool f32, int rows, int col
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+std::atomic<long long> g_wait_limit{DRAIN_LIMIT_CYCLES};
+
 int tc_bn(int nmax) {
   int BN = ((nmax + 15) / 16) * 16;
   return BN > 256 ? 256 : BN;
@@ -433,6 +470,7 @@ cudaError_t gemm_tc_grouped(const TcSpec* spec, int nprob, int32_t* status, cuda
   a.nprob = nprob;
   a.BN = BN;
   a.tmem_cols = cols;
+  a.wait_limit = g_wait_limit.load(std::memory_order_relaxed);
   a.status = status;
   int total = 0;
   for (int i = 0; i < 2; ++i) {
@@ -479,3 +517,8 @@ cudaError_t gemm_tc(int M, int N, int K, const void* A, int lda, const void* B, 
 }
 
 }  // namespace brisk
+
+extern "C" int64_t brisk_set_wait_limit(int64_t cycles) {
+  const long long v = cycles > 0 ? (long long)cycles : brisk::DRAIN_LIMIT_CYCLES;
+  return (int64_t)brisk::g_wait_limit.exchange(v);
+}

@@ -98,3 +98,15 @@ def test_binding_refuses_to_run_without_the_library(tmp_path, monkeypatch):
     monkeypatch.setattr(brisk, "LIB_PATH", str(tmp_path / "missing.so"))
     with pytest.raises(RuntimeError):
         brisk.lib()
+
+
+def test_wait_limit_setter_returns_the_previous_limit(B):
+    default = 4000000000
+    prev = B.set_wait_limit(1234)
+    try:
+        assert prev == default
+        assert B.set_wait_limit(0) == 1234          # 0 restores the default
+        assert B.set_wait_limit(-5) == default
+        assert B.set_wait_limit(99) == default
+    finally:
+        B.set_wait_limit(0)
