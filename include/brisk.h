@@ -157,8 +157,9 @@ brisk_status brisk_topk_candidates(const brisk_dims *dims, const void *logits_q,
  * present on every GPU that loads the library until the process exits, and allocates nothing.
  *  - Returns BRISK_ERR_UNSUPPORTED when the problem needs more than that array holds (its
  *    per-row arrival counters and per-chunk partial results grow with B*L and K).
- *  - The first call on a device looks up the array's device address (cudaGetSymbolAddress);
- *    make that first call before any stream capture.
+ *  - The first call in a CUDA context looks up the array's device address there
+ *    (cudaGetSymbolAddress) and keeps it for that context; after a device reset (a new context)
+ *    the next call looks it up again. Make the first call on a device before any stream capture.
  *  - Every call on a device shares the one array; calls that can overlap on the GPU (other
  *    streams, other host threads) race and must be serialised by the caller.
  *  - Device-side problems are not reported through a status word: a row without a finite
@@ -204,9 +205,10 @@ brisk_status brisk_verify_block(const brisk_dims *dims, const void *logits_p,
  * batch is small enough that the proposal rows are swept in several chunks each, the critical
  * path runs on `stream` itself and the verifier sweep starts after the proposal sweep. The call
  * only enqueues work and the results are ordered on `stream` (the side streams fork from and
- * join back to it, also under graph capture). The first call on a device creates the side streams and their events: make it
- * before any stream capture. Calls from several host threads are serialised while they enqueue.
- * `ev` may be NULL. */
+ * join back to it, also under graph capture). The first call in a CUDA context creates the side
+ * streams and their events: make it before any stream capture. Calls from several host threads
+ * are serialised while they enqueue, and brisk_tail_graph_create holds that serialisation for
+ * the whole of its capture. `ev` may be NULL. */
 brisk_status brisk_decode_tail(const brisk_dims *dims, const brisk_params *params,
                                const void *tables, const brisk_tail_io *io, int32_t select_mode,
                                int32_t verify_mode, void *workspace, const brisk_events *ev,
@@ -242,6 +244,18 @@ int32_t brisk_kernels_per_tail(const brisk_dims *dims);
  * outside [0, V) (BRISK_ERR_INVALID_ARG; the id is replaced by 0 so that nothing reads out of
  * bounds). With clear != 0 the word is reset to BRISK_OK afterwards. */
 brisk_status brisk_last_device_status(void *workspace, int32_t clear, void *stream);
+
+/* Sets the limit, in SM clock cycles, of the bounded device-side waits (the tensor-core
+ * products' pipeline and accumulator waits, which no other kernel has: the sweep, corrector and
+ * verification kernels never wait on another CTA or on a copy). cycles <= 0 restores the default
+ * of 4e9 cycles (about 2 s). Returns the previous limit. The value is read when a launch is
+ * enqueued and passed to the kernel (a captured graph keeps the value it was captured with); it
+ * is process-wide. When a wait gives up, the call records BRISK_ERR_TIMEOUT in the device status,
+ * its outputs are undefined, and the kernel still waits (up to the default limit) for the copies
+ * and tensor-core operations it started before it frees its resources and returns, so the CUDA
+ * context stays usable. A short limit makes waits give up while their data is still arriving:
+ * tests of the failure path use it. No counterpart in the paper (failure detection). */
+int64_t brisk_set_wait_limit(int64_t cycles);
 
 /* Human-readable name of a status code (static storage). */
 const char *brisk_status_string(brisk_status status);

@@ -76,6 +76,7 @@ _SIGS = [
     ("brisk_kernels_per_tail", ctypes.c_int32, [ctypes.POINTER(Dims)]),
     ("brisk_last_device_status", ctypes.c_int, [_vp, ctypes.c_int32, _vp]),
     ("brisk_status_string", ctypes.c_char_p, [ctypes.c_int]),
+    ("brisk_set_wait_limit", ctypes.c_int64, [ctypes.c_int64]),
     ("brisk_acceptance_counts", ctypes.c_int, [_vp, ctypes.c_int32, ctypes.c_int32, _vp, _vp]),
     ("brisk_acceptance_weights", ctypes.c_int,
      [ctypes.c_int32, _vp, _vp, _vp, ctypes.c_double, _vp, _vp, _vp]),
@@ -108,6 +109,12 @@ def lib():
             f.argtypes = args
         _lib = h
     return _lib
+
+
+def set_wait_limit(cycles: int) -> int:
+    """Limit (SM cycles) of the library's bounded device-side waits; <= 0 restores the default.
+    Returns the previous limit."""
+    return int(lib().brisk_set_wait_limit(int(cycles)))
 
 
 def status_string(s: int) -> str:

@@ -1,4 +1,7 @@
 // C ABI of the decode tail: argument checks, workspace and table layouts, launches.
+#include <cuda.h>
+
+#include <deque>
 #include <mutex>
 #include <string.h>
 
@@ -189,22 +192,31 @@ brisk_status hidden_products(const brisk_dims* d, const brisk_params* p, const v
   return BRISK_OK;
 }
 
-// A side stream per device (created on the first fused call on that device) and the events that
-// fork work onto it and join it back, so that one call can run independent stages concurrently.
+// Side streams per CUDA context (created on the first fused call in that context, so a device
+// reset gets new ones) and the events that fork work onto them and join it back, so that one
+// call can run independent stages concurrently.
 struct SideStream {
+  unsigned long long ctx = 0;   // id of the context the streams belong to
   cudaStream_t hi = nullptr;    // highest priority: the hidden-state products
   cudaStream_t mid = nullptr;   // middle priority: proposal sweep, corrector, verification
   cudaStream_t lo = nullptr;    // lowest priority: the verifier-row sweep
   cudaEvent_t ev[5] = {};
 };
-constexpr int MAX_DEVICES = 256;
-std::mutex g_side_mu;
-SideStream g_side[MAX_DEVICES];
+std::deque<SideStream> g_side;   // guarded by side_stream_mutex(); elements never move
 
+// The current context's side streams; the caller holds side_stream_mutex().
 SideStream* side_stream() {
-  int dev = -1;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= MAX_DEVICES) return nullptr;
-  SideStream& ss = g_side[dev];
+  unsigned long long ctx = 0;
+  if (!brisk::current_context_id(&ctx)) return nullptr;
+  SideStream* found = nullptr;
+  for (auto& e : g_side)
+    if (e.ctx == ctx) found = &e;
+  if (!found) {
+    g_side.emplace_back();
+    found = &g_side.back();
+    found->ctx = ctx;
+  }
+  SideStream& ss = *found;
   if (!ss.hi) {
     int least = 0, greatest = 0;
     if (cudaDeviceGetStreamPriorityRange(&least, &greatest) != cudaSuccess) return nullptr;
@@ -250,6 +262,34 @@ ScanArgs scan_args(const brisk_dims* d, const brisk_params* p, const void* table
 }
 
 }  // namespace
+
+std::mutex& brisk::side_stream_mutex() {
+  static std::mutex mu;
+  return mu;
+}
+
+bool brisk::current_context_id(unsigned long long* id) {
+  using GetCurrent = CUresult (*)(CUcontext*);
+  using GetId = CUresult (*)(CUcontext, unsigned long long*);
+  static GetCurrent get_current = nullptr;
+  static GetId get_id = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess && q == cudaDriverEntryPointSuccess)
+      get_current = reinterpret_cast<GetCurrent>(p);
+    p = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess && q == cudaDriverEntryPointSuccess)
+      get_id = reinterpret_cast<GetId>(p);
+  });
+  if (!get_current || !get_id) return false;
+  CUcontext c = nullptr;
+  if (get_current(&c) != CUDA_SUCCESS || !c) return false;
+  return get_id(c, id) == CUDA_SUCCESS;
+}
 
 extern "C" {
 
@@ -433,6 +473,19 @@ brisk_status brisk_verify_block(const brisk_dims* d, const void* logits_p, const
 brisk_status brisk_decode_tail(const brisk_dims* d, const brisk_params* p, const void* tables,
                                const brisk_tail_io* io, int32_t select_mode, int32_t verify_mode,
                                void* ws, const brisk_events* ev, void* stream) {
+  std::lock_guard<std::mutex> lock(side_stream_mutex());
+  return brisk::decode_tail_locked(d, p, tables, io, select_mode, verify_mode, ws, ev, stream);
+}
+
+}  // extern "C"
+
+// The body of brisk_decode_tail; the caller holds side_stream_mutex() (brisk_tail_graph_create
+// holds it from the start of its capture to the end, so that no other thread's work lands on
+// the side streams while they belong to the capture).
+brisk_status brisk::decode_tail_locked(const brisk_dims* d, const brisk_params* p,
+                                       const void* tables, const brisk_tail_io* io,
+                                       int32_t select_mode, int32_t verify_mode, void* ws,
+                                       const brisk_events* ev, void* stream) {
   if (!dims_ok(d) || !params_ok(p) || !tables || !io || !ws || !aligned(ws, ALIGN) ||
       !aligned(tables, ALIGN))
     return BRISK_ERR_INVALID_ARG;
@@ -472,7 +525,6 @@ brisk_status brisk_decode_tail(const brisk_dims* d, const brisk_params* p, const
   // which saves the extra fork and keeps the SMs free for the corrector's start; the products,
   // on the critical path there, use narrow tiles (more CTAs).
   const bool overlap = w.nchunk_q == 1;
-  std::lock_guard<std::mutex> lock(g_side_mu);
   SideStream* ss = side_stream();
   if (!ss) return BRISK_ERR_CUDA;
   cudaStream_t m = overlap ? ss->mid : st;
@@ -551,6 +603,8 @@ brisk_status brisk_decode_tail(const brisk_dims* d, const brisk_params* p, const
   }
   return BRISK_OK;
 }
+
+extern "C" {
 
 int32_t brisk_kernels_per_tail(const brisk_dims* dims) {
   if (!dims_ok(dims)) return 0;

@@ -331,4 +331,19 @@ cudaError_t launch_replay(const ReplayArgs& a, cudaStream_t stream);
 size_t scan_smem_bytes(int L, int K, int S, int V);
 cudaError_t launch_scan(const ScanArgs& a, cudaStream_t stream);
 
+// ---------------------------------------------------------------- contexts
+// Unique id of the CUDA context current on this thread (cuCtxGetId; ids are never reused, so a
+// device reset, which creates a new context, gives a new id). False when no context is current
+// or the driver entry points are unavailable.
+bool current_context_id(unsigned long long* id);
+
+// ---------------------------------------------------------------- fused tail
+// Serialises the use of the library's side streams: held while one call enqueues on them, and
+// by graph creation from the start of its capture to the end.
+std::mutex& side_stream_mutex();
+// brisk_decode_tail with side_stream_mutex() already held by the caller.
+brisk_status decode_tail_locked(const brisk_dims* d, const brisk_params* p, const void* tables,
+                                const brisk_tail_io* io, int32_t select_mode, int32_t verify_mode,
+                                void* ws, const brisk_events* ev, void* stream);
+
 }  // namespace brisk

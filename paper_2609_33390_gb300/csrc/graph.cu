@@ -29,12 +29,16 @@ extern "C" brisk_status brisk_tail_graph_create(const brisk_dims* dims, const br
   if (cudaStreamSynchronize(st) != cudaSuccess) return BRISK_ERR_CUDA;
   brisk_graph* g = new (std::nothrow) brisk_graph();
   if (!g) return BRISK_ERR_CUDA;
+  // The side streams belong to the capture from the call's first fork until the end of the
+  // capture: hold their lock over the whole of it, so that another thread's call cannot enqueue
+  // on them in between (its work would land in this graph, or break the capture).
+  std::lock_guard<std::mutex> lock(brisk::side_stream_mutex());
   if (cudaStreamBeginCapture(st, cudaStreamCaptureModeThreadLocal) != cudaSuccess) {
     delete g;
     return BRISK_ERR_CUDA;
   }
-  s = brisk_decode_tail(dims, params, tables, io, select_mode, verify_mode, workspace, nullptr,
-                        stream);
+  s = brisk::decode_tail_locked(dims, params, tables, io, select_mode, verify_mode, workspace,
+                                nullptr, stream);
   const cudaError_t ec = cudaStreamEndCapture(st, &g->graph);
   if (s != BRISK_OK || ec != cudaSuccess ||
       cudaGraphInstantiate(&g->exec, g->graph, 0) != cudaSuccess) {

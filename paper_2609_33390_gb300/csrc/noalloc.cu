@@ -21,25 +21,31 @@ namespace {
 constexpr size_t NOALLOC_SCRATCH_BYTES = size_t(4) << 20;
 static __device__ __align__(256) unsigned char g_noalloc_scratch[NOALLOC_SCRATCH_BYTES];
 
-constexpr int NOALLOC_MAX_DEVICES = 256;
 std::mutex g_noalloc_mu;
-void* g_noalloc_addr[NOALLOC_MAX_DEVICES] = {};
+std::vector<std::pair<unsigned long long, void*>> g_noalloc_addr;   // (context id, address)
 
 inline size_t up256(size_t x) { return (x + 255) / 256 * 256; }
 
-// Device address of the scratch array on the current device. The first call on a
-// device looks it up (cudaGetSymbolAddress) and caches it; host code must never
-// hand the array's own name to a kernel, since on the host it is only a stand-in.
+// Device address of the scratch array in the current CUDA context. The first call in a
+// context looks it up (cudaGetSymbolAddress, which also loads the library's module there) and
+// caches it under the context's id; a device reset makes a new context with a new id, in which
+// the address is looked up again, so a stale address is never used. Host code must never hand
+// the array's own name to a kernel, since on the host it is only a stand-in.
 void* noalloc_scratch_address() {
-  int dev = -1;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= NOALLOC_MAX_DEVICES) return nullptr;
-  std::lock_guard<std::mutex> lock(g_noalloc_mu);
-  if (!g_noalloc_addr[dev]) {
+  unsigned long long ctx = 0;
+  if (!current_context_id(&ctx)) {
+    // no context current yet: the lookup below initialises the device's primary context
     void* p = nullptr;
     if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || !p) return nullptr;
-    g_noalloc_addr[dev] = p;
+    if (!current_context_id(&ctx)) return nullptr;
   }
-  return g_noalloc_addr[dev];
+  std::lock_guard<std::mutex> lock(g_noalloc_mu);
+  for (const auto& e : g_noalloc_addr)
+    if (e.first == ctx) return e.second;
+  void* p = nullptr;
+  if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || !p) return nullptr;
+  g_noalloc_addr.emplace_back(ctx, p);
+  return p;
 }
 
 }  // namespace
