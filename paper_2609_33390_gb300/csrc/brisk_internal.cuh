@@ -179,6 +179,60 @@ inline cudaError_t prefer_carveout(Kernel kernel, int kb) {
   return prefer_carveout_fn(reinterpret_cast<const void*>(kernel), kb);
 }
 
+// ---------------------------------------------------------------- mbarriers and bulk copies
+// Bounded waits: a wait gives up after a limit of SM cycles (wait_limit_cycles(), set by
+// brisk_set_wait_limit and passed to kernels as an argument); the drain of copies still in
+// flight after a give-up is bounded by the default limit.
+constexpr long long DRAIN_LIMIT_CYCLES = 4000000000ll;  // about 2 s of SM clock
+constexpr long long SHORT_WAIT_CYCLES = 1ll << 20;      // below this, waits poll without suspending
+long long wait_limit_cycles();
+
+__device__ __forceinline__ uint32_t su32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(su32(bar)), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(su32(bar)), "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(su32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+// Non-blocking test of the phase with the given parity (never suspends the thread).
+__device__ __forceinline__ bool mbar_test(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(su32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+// Wait for a phase that is known to complete (the drain after a give-up), bounded by the
+// default limit.
+__device__ __forceinline__ void mbar_drain(uint64_t* bar, uint32_t parity) {
+  const long long t0 = clock64();
+  while (!mbar_try_wait(bar, parity) && clock64() - t0 < DRAIN_LIMIT_CYCLES) {
+  }
+}
+// Orders this thread's earlier shared-memory accesses before later async-proxy (TMA, bulk copy)
+// accesses of the same memory.
+__device__ __forceinline__ void fence_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
 __device__ __forceinline__ void set_status(int32_t* status, int code) {
   if (status) atomicCAS(status, 0, code);
 }

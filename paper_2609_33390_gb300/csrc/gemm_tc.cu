@@ -29,43 +29,7 @@ constexpr int TC_BM = 128;
 constexpr int TC_BK = 64;               // one 128-byte swizzle row of bf16
 constexpr int TC_STAGES_MAX = 4;
 constexpr int TC_THREADS = 128;
-constexpr long long DRAIN_LIMIT_CYCLES = 4000000000ll;  // about 2 s of SM clock per drain wait
-constexpr long long SHORT_WAIT_CYCLES = 1ll << 20;      // below this, waits poll without suspending
 
-__device__ __forceinline__ uint32_t su32(const void* p) {
-  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
-
-__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
-  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(su32(bar)), "r"(count) : "memory");
-}
-__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
-  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(su32(bar)), "r"(bytes)
-               : "memory");
-}
-__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
-  uint32_t ok;
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-      "selp.u32 %0, 1, 0, p;\n\t}"
-      : "=r"(ok)
-      : "r"(su32(bar)), "r"(parity)
-      : "memory");
-  return ok != 0;
-}
-// Non-blocking test of the phase with the given parity (never suspends the thread).
-__device__ __forceinline__ bool mbar_test(uint64_t* bar, uint32_t parity) {
-  uint32_t ok;
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-      "selp.u32 %0, 1, 0, p;\n\t}"
-      : "=r"(ok)
-      : "r"(su32(bar)), "r"(parity)
-      : "memory");
-  return ok != 0;
-}
 // Bounded wait for the phase with the given parity; false on expiry (more than `limit` SM
 // cycles) or abort. With a long limit the thread may suspend in try_wait and the cycle counter
 // and the abort flag are read every 64 polls; a short limit (tests of the failure path) polls
@@ -86,13 +50,7 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volati
     if ((n & 63) == 0 && (*abort_flag || clock64() - t0 > limit)) return false;
   }
 }
-// Wait for a phase that is known to complete (the drain after an abort), bounded by the
-// default limit.
-__device__ __forceinline__ void mbar_drain(uint64_t* bar, uint32_t parity) {
-  const long long t0 = clock64();
-  while (!mbar_try_wait(bar, parity) && clock64() - t0 < DRAIN_LIMIT_CYCLES) {
-  }
-}
+
 __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, uint64_t* bar, int x,
                                             int y) {
   asm volatile(
@@ -117,10 +75,6 @@ __device__ __forceinline__ void bulk_wait_read(int n) {
   else asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
 }
 __device__ __forceinline__ void bulk_wait0() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
-// Makes this thread's shared-memory writes visible to the async (TMA) proxy.
-__device__ __forceinline__ void fence_async_smem() {
-  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-}
 __device__ __forceinline__ void tmem_alloc(uint32_t* slot, uint32_t ncols) {
   asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(su32(slot)),
                "r"(ncols)
@@ -438,6 +392,12 @@ bool make_out_map(CUtensorMap* map, const void* ptr, bool f32, int rows, int col
 
 std::atomic<long long> g_wait_limit{DRAIN_LIMIT_CYCLES};
 
+}  // namespace
+
+long long wait_limit_cycles() { return g_wait_limit.load(std::memory_order_relaxed); }
+
+namespace {
+
 int tc_bn(int nmax) {
   int BN = ((nmax + 15) / 16) * 16;
   return BN > 256 ? 256 : BN;
@@ -470,7 +430,7 @@ cudaError_t gemm_tc_grouped(const TcSpec* spec, int nprob, int32_t* status, cuda
   a.nprob = nprob;
   a.BN = BN;
   a.tmem_cols = cols;
-  a.wait_limit = g_wait_limit.load(std::memory_order_relaxed);
+  a.wait_limit = wait_limit_cycles();
   a.status = status;
   int total = 0;
   for (int i = 0; i < 2; ++i) {

@@ -763,9 +763,8 @@ size_t scan_smem_bytes(int L, int K, int S, int V) {
   return smem_layout(L, K, S, V, nullptr, nullptr);
 }
 
-template <int NP, int CMC>
+template <int NP, int CMC, int NW = CORR_WARPS>
 cudaError_t launch_corrector(const ScanArgs& a, cudaStream_t stream) {
-  constexpr int NW = CORR_WARPS;
   const size_t smem = corr_layout(a.L, a.K, a.S, NW, nullptr, nullptr);
   cudaError_t e = cudaFuncSetAttribute(corrector_kernel<NW, NP, CMC>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
@@ -778,10 +777,15 @@ cudaError_t launch_corrector(const ScanArgs& a, cudaStream_t stream) {
 // The corrector (do_select) or the verification (do_verify) for every sequence.
 cudaError_t launch_scan(const ScanArgs& a, cudaStream_t stream) {
   if (a.do_select) {
-    // 4-element chunks per lane: S / 4 chunks over CORR_WARPS * 32 lanes (S <= 1024)
+    // 4-element chunks per lane: S / 4 chunks over the CTA's lanes. A state wider than four
+    // warps' chunks (S > 512, up to 1024) takes eight warps, one chunk a lane, rather than two
+    // chunks a lane: the next position's residual rows then fit the register pipeline, and each
+    // SM sub-partition has two warps of the sequence to issue from (large_vocab, S = 1024,
+    // K = 16: products and corrector 535 -> 284 us, step 856 -> 604 us).
     if (a.S > 4 * 32 * CORR_WARPS) {
-      if (a.K <= 8) return launch_corrector<8, 2>(a, stream);
-      return a.K <= 16 ? launch_corrector<16, 2>(a, stream) : launch_corrector<32, 2>(a, stream);
+      if (a.K <= 8) return launch_corrector<8, 1, 2 * CORR_WARPS>(a, stream);
+      return a.K <= 16 ? launch_corrector<16, 1, 2 * CORR_WARPS>(a, stream)
+                       : launch_corrector<32, 1, 2 * CORR_WARPS>(a, stream);
     }
     if (a.K <= 8) return launch_corrector<8, 1>(a, stream);
     return a.K <= 16 ? launch_corrector<16, 1>(a, stream) : launch_corrector<32, 1>(a, stream);

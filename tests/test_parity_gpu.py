@@ -72,6 +72,13 @@ SMALL = [
     ("k_equals_v", dict(B=2, L=4, V=8, d=16, K=8, r=16, select_mode="sample",
                         verify_mode="stochastic")),
     ("long_block", dict(B=1, L=64, V=1500, d=32, K=8, r=16)),
+    # states wider than 512 (eight warps a sequence), every K class of that kernel; weights of
+    # std 0.06 keep the refined scores O(10) as in the workloads (at 0.2 they reach ~2800, where
+    # fp32 rounding alone is ~1e-5 relative, beyond the 1e-3 absolute bound)
+    ("wide_state_k8_sample", dict(B=2, L=5, V=2000, d=64, K=8, r=512, select_mode="sample",
+                                  verify_mode="stochastic", weight_std=0.06)),
+    ("wide_state_k16", dict(B=2, L=7, V=2500, d=64, K=16, r=384, weight_std=0.06)),
+    ("wide_state_k32", dict(B=2, L=6, V=3000, d=64, K=32, r=512, weight_std=0.06)),
 ]
 
 
