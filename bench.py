@@ -461,9 +461,21 @@ def run_ours(args):
         e2e.pop("_tokens", None)
         e2e.pop("_seconds", None)
 
+    # acceptance of the timed blocks with the corrector's gate closed (base ranking), after
+    # the timed region, on the same blocks and anchors
+    alpha = tail.params.alpha
+    tail.params.alpha = float("-inf")
+    acc_off = 0
+    for s in range(args.warmup, nsteps):
+        blk = pool[s % pool_n]
+        x0 = blk["x0"] if s == 0 else outs[s - 1]["next_anchor"]
+        acc_off += int(tail.tail(blk, sm, vm, x0=x0)["accepted_len"].sum())
+    tail.params.alpha = alpha
+
     if rank != 0:
         return 0
     graph_loop = run_graph_loop(dev)
+    per_config = None if args.no_per_config else run_per_config(dev, args.per_config_steps)
     cpu = None
     if not args.no_cpu_baseline:
         cpu = cpu_baseline_entry(list(range(CPU_SAMPLE_SEQS)))
@@ -492,6 +504,7 @@ def run_ours(args):
         "committed_tokens_per_s": committed_all / elapsed_max,
         "host_enqueue_us_per_step": 1e6 * host_enqueue_s / args.steps,
         "accepted_per_sequence_block": tokens / (wl.B * world * args.steps),
+        "accepted_per_sequence_block_corrector_off": acc_off / (wl.B * args.steps),
         "acceptance_profile": {"a": [round(x, 4) for x in prof_a[:8]],
                                "positions_shown": min(8, wl.L),
                                "tpf_unit_cost": prof_tpf,
@@ -499,6 +512,7 @@ def run_ours(args):
                                "tpf_isd_eq8": isd_tpf,
                                "w_bar_isd_eq8": [round(x, 4) for x in isd_w[:8]]},
         "graph_loop": graph_loop,
+        "per_config": per_config,
         "distill_loss_us": distill_us,
         "replay": {"first_breakers": n_fb,
                    "intervention_rate_at_breakers": n_int / max(1, n_fb),
@@ -563,6 +577,84 @@ def run_graph_loop(dev, blocks=30):
                           "buffer sets, overlapped with the running block",
             "kernels_per_block": brisk.kernels_per_tail(tail.dims),
             "accepted_last_block": acc}
+
+
+PER_CONFIG = ("tiny", "single", "batched_stochastic", "large_vocab")
+L2_FLUSH_BYTES = 256 << 20   # twice the 129 MB L2
+
+
+def run_per_config(dev, steps, names=PER_CONFIG, pool_n=3):
+    """Every other workload configuration at its full size, outside the headline's timed region:
+    per step (a fused decode-tail call, CUDA events on its stream, L2 flushed by a 256 MB write
+    before each step and outside the events) the device time, the span of the two sweep launches
+    (events the library records around them) and the accepted tokens; then the same blocks with
+    the corrector's gate closed (alpha = -inf: the base ranking, rank 0 under greedy Select), for
+    the acceptance the corrector changes."""
+    import torch
+    from paper_2609_33390_gb300 import brisk, synth
+    peak, peak_src = measured_peaks()
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream()
+    res = {}
+    for name in names:
+        wl = synth.WORKLOADS[name]
+        tail = brisk.DecodeTail.for_workload(wl, synth.make_weights(wl, dev), dev)
+        tail.prepare()
+        pool = [synth.make_block(wl, dev, block=j) for j in range(pool_n)]
+        sm, vm = brisk.mode_ids(wl.select_mode, wl.verify_mode)
+        nsteps = 3 + steps
+        outs = [tail.alloc_outputs(full=False) for _ in range(nsteps)]
+        evs = [tuple(torch.cuda.Event(enable_timing=True) for _ in range(6)) for _ in range(nsteps)]
+        for ev in evs:
+            for e in ev:
+                e.record(stream)
+        torch.cuda.synchronize()
+        for s in range(nsteps):
+            blk = pool[s % pool_n]
+            x0 = blk["x0"] if s == 0 else outs[s - 1]["next_anchor"]
+            flush.zero_()
+            evs[s][4].record(stream)
+            tail.tail(blk, sm, vm, out=outs[s], x0=x0, events=evs[s][:4])
+            evs[s][5].record(stream)
+        torch.cuda.synchronize()
+        st = tail.device_status()
+        if st != brisk.OK:
+            raise RuntimeError(f"{name}: device status {brisk.status_string(st)}")
+        timed = range(3, nsteps)
+        step_ms = [evs[s][4].elapsed_time(evs[s][5]) for s in timed]
+        span_ms = [sweep_span_ms(*evs[s][:4]) for s in timed]
+        acc = sum(int(outs[s]["accepted_len"].sum()) for s in timed)
+        # the same blocks and anchors with the gate closed
+        alpha = tail.params.alpha
+        tail.params.alpha = float("-inf")
+        acc_off = 0
+        for s in timed:
+            blk = pool[s % pool_n]
+            x0 = blk["x0"] if s == 0 else outs[s - 1]["next_anchor"]
+            o = tail.tail(blk, sm, vm, x0=x0)
+            acc_off += int(o["accepted_len"].sum())
+        tail.params.alpha = alpha
+        torch.cuda.synchronize()
+        sweep_s = statistics.mean(span_ms) / 1000.0
+        gbs = wl.sweep_bytes() / sweep_s / 1e9
+        n_blocks = wl.B * steps
+        res[name] = {
+            "B": wl.B, "L": wl.L, "V": wl.V, "d": wl.d, "K": wl.K, "r": wl.r,
+            "select": wl.select_mode, "verify": wl.verify_mode, "steps": steps,
+            "us_per_step_mean": 1000.0 * statistics.mean(step_ms),
+            "us_per_step_median": 1000.0 * statistics.median(step_ms),
+            "accepted_tokens_per_s": acc / (sum(step_ms) / 1000.0),
+            "sweep_bytes": wl.sweep_bytes(), "sweep_span_us": 1e6 * sweep_s,
+            "sweep_gbs": gbs, "sweep_frac_of_peak": gbs / peak, "peak_source": peak_src,
+            "sweep_frac_of_nameplate_8tbs": gbs / NAMEPLATE_HBM_GBS,
+            "sweep_share_of_step": statistics.mean(span_ms) / statistics.mean(step_ms),
+            "accepted_per_sequence_block": acc / n_blocks,
+            "accepted_per_sequence_block_corrector_off": acc_off / n_blocks,
+            "l2": "256 MB written before every step, outside its events",
+        }
+        del tail, pool, outs
+        torch.cuda.empty_cache()
+    return res
 
 
 def run_e2e(args, tail, pool, wl, sm, vm, dev):
@@ -639,6 +731,9 @@ def main(argv=None):
     ap.add_argument("--pool", type=int, default=16, help="distinct pre-generated blocks cycled")
     ap.add_argument("--e2e-steps", type=int, default=20)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-per-config", action="store_true",
+                    help="skip the measurements of the other four workload configurations")
+    ap.add_argument("--per-config-steps", type=int, default=20)
     ap.add_argument("--profile", default=None, help="workload name: short untimed run for ncu")
     args = ap.parse_args(argv)
     args.warmup = max(3, args.warmup)   # at least 3 untimed warm-up steps
