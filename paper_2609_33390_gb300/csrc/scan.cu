@@ -21,8 +21,12 @@ namespace brisk {
 
 namespace {
 
-constexpr int SCAN_THREADS = 128;
-constexpr int SCAN_WARPS = SCAN_THREADS / 32;
+// Verification CTA: 128 threads, or 512 under stochastic verification, where a rejection
+// resamples from a residual over the whole vocabulary row (a 126464-entry row: 112 us on 128
+// threads with element loads and the precise exponential, a few us with 512 threads, vector
+// loads and the hardware one).
+constexpr int VERIFY_THREADS = 128;
+constexpr int VERIFY_THREADS_MAX = 512;
 
 struct Smem {
   int* cid;        // [L][K]
@@ -141,17 +145,36 @@ __device__ __forceinline__ float proposal_mass(const float* ref, int K, int mode
   return expf(ref[r] - mx) / tot;
 }
 
-// Residual R(v) = max(0, p(v) - pi(v)) of the 8 ids [v0, v0+8) owned by this lane.
-// Lanes k < K hold candidate k: (cand_id, cand_mass).
+// Residual R(v) = max(0, p(v) - pi(v)) of the 8 ids [v0, v0+8) owned by this lane, with
+// p(v) = 2^(l(v) log2 e - lse log2 e) on the hardware exponential (v0 is a multiple of 8, so a
+// 16-byte-aligned row gives aligned 16-byte vector loads; ragged ends and unaligned rows take
+// element loads). Lanes k < K hold candidate k: (cand_id, cand_mass).
 __device__ __forceinline__ void residual8(const void* rowp, int dt, int V, float lse, int v0,
                                          int blk0, int cand_id, float cand_mass, int K,
                                          float (&R)[8]) {
   const int lane = threadIdx.x & 31;
+  const float nlb = -lse * LOG2E;
+  float l[8];
+  const bool vec = v0 + 8 <= V && (reinterpret_cast<uintptr_t>(rowp) & 15u) == 0;
+  if (vec && dt == BRISK_DT_BF16) {
+    unpack(__ldg(reinterpret_cast<const uint4*>(reinterpret_cast<const __nv_bfloat16*>(rowp) + v0)),
+           l, __nv_bfloat16());
+  } else if (vec) {
+    const uint4* q = reinterpret_cast<const uint4*>(reinterpret_cast<const float*>(rowp) + v0);
+    float a[4], b[4];
+    unpack(__ldg(q), a, 0.f);
+    unpack(__ldg(q + 1), b, 0.f);
 #pragma unroll
-  for (int e = 0; e < 8; ++e) {
-    const int v = v0 + e;
-    R[e] = (v < V) ? expf(load_logit(rowp, dt, (size_t)v) - lse) : 0.f;
+    for (int e = 0; e < 4; ++e) {
+      l[e] = a[e];
+      l[4 + e] = b[e];
+    }
+  } else {
+#pragma unroll
+    for (int e = 0; e < 8; ++e) l[e] = v0 + e < V ? load_logit(rowp, dt, (size_t)(v0 + e)) : -INFINITY;
   }
+#pragma unroll
+  for (int e = 0; e < 8; ++e) R[e] = ex2(fmaf(l[e], LOG2E, nlb));
   const bool mine = lane < K && cand_id >= blk0 && cand_id < blk0 + RES_BLOCK;
   unsigned mask = __ballot_sync(FULL_MASK, mine);
   while (mask) {
@@ -184,7 +207,7 @@ __device__ int residual_sample(const Smem& sm, const void* rowp, int dt, int V, 
     else cand_mass = proposal_mass(ref, K, select_mode, lane);
   }
   // pass 1: block sums (blocks interleaved over warps)
-  for (int blk = warp; blk < nblk; blk += SCAN_WARPS) {
+  for (int blk = warp; blk < nblk; blk += (int)(blockDim.x >> 5)) {
     const int blk0 = blk * RES_BLOCK;
     float R[8];
     residual8(rowp, dt, V, lse, blk0 + lane * 8, blk0, cand_id, cand_mass, K, R);
@@ -306,7 +329,7 @@ __device__ void verify_sequence(const ScanArgs& a, const Smem& sm, int b) {
   const int L = a.L, K = a.K;
   if (tid == 0) sm.imisc[2] = L;
   __syncthreads();
-  for (int t = tid; t < L; t += SCAN_THREADS) {
+  for (int t = tid; t < L; t += (int)blockDim.x) {
     const size_t bi = (size_t)b * L + t;
     const int x = sm.sel[t];
     bool ok;
@@ -342,13 +365,13 @@ __device__ void verify_sequence(const ScanArgs& a, const Smem& sm, int b) {
     a.correction[b] = (j < L) ? corr : -1;
     if (a.next_anchor) a.next_anchor[b] = (j < L) ? corr : sm.sel[L - 1];
   }
-  for (int t = tid; t < L; t += SCAN_THREADS)
+  for (int t = tid; t < L; t += (int)blockDim.x)
     a.out_tokens[(size_t)b * L + t] = t < j ? sm.sel[t] : (t == j ? corr : -1);
 }
 
 // Verification of one sequence per CTA (Sec. 3.1; Sec. 3.3; App. B Eq. 6), reading the
 // selections and refined scores the corrector wrote.
-__global__ void __launch_bounds__(SCAN_THREADS)
+__global__ void __launch_bounds__(VERIFY_THREADS_MAX)
 verify_kernel(const __grid_constant__ ScanArgs a) {
   extern __shared__ __align__(16) char smem_raw[];
   Smem sm;
@@ -359,20 +382,21 @@ verify_kernel(const __grid_constant__ ScanArgs a) {
   const size_t bL = (size_t)b * L;
   // Ids are gathered with below, so out-of-range ones (a row with no finite logit leaves
   // placeholder ids; caller-provided ids may be anything) are replaced by 0 and reported.
-  for (int e = tid; e < L * K; e += SCAN_THREADS) {
+  const int nt = (int)blockDim.x;
+  for (int e = tid; e < L * K; e += nt) {
     int c = a.cand_ids[bL * K + e];
     if (c < 0 || c >= V) { set_status(a.status, BRISK_ERR_NUMERIC); c = 0; }
     sm.cid[e] = c;
     sm.ref[e] = a.refined[bL * K + e];
   }
-  for (int e = tid; e < L; e += SCAN_THREADS) {
+  for (int e = tid; e < L; e += nt) {
     int x = a.sel_tokens[bL + e];
     if (x < 0 || x >= V) { set_status(a.status, BRISK_ERR_INVALID_ARG); x = 0; }
     sm.sel[e] = x;
   }
   __syncthreads();
   // each selection's rank in its candidate list
-  for (int i = tid; i < L; i += SCAN_THREADS) {
+  for (int i = tid; i < L; i += nt) {
     int r = 0;
     for (int k = 0; k < K; ++k)
       if (sm.cid[i * K + k] == sm.sel[i]) { r = k; break; }
@@ -795,7 +819,8 @@ cudaError_t launch_scan(const ScanArgs& a, cudaStream_t stream) {
                                        (int)smem);
   if (e == cudaSuccess) e = prefer_carveout(verify_kernel, CARVEOUT_SMALL_KB);
   if (e != cudaSuccess) return e;
-  verify_kernel<<<a.B, SCAN_THREADS, smem, stream>>>(a);
+  const int threads = a.verify_mode == BRISK_VERIFY_STOCHASTIC ? VERIFY_THREADS_MAX : VERIFY_THREADS;
+  verify_kernel<<<a.B, threads, smem, stream>>>(a);
   return cudaGetLastError();
 }
 
