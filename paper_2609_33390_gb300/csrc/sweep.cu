@@ -342,19 +342,27 @@ __device__ __forceinline__ void publish_partial(const SweepSeg& sg, int row, int
   if (prev != parts - 1) return;
   __threadfence();
 
-  // last part of the row: merge the partials in part order
+  // last part of the row: merge the partials in part order, the lists of MERGE_BATCH parts
+  // loaded at once (one L2 round trip per batch instead of one per part)
+  constexpr int MERGE_BATCH = 8;
   wv = -INFINITY;
   wi = INVALID_ID;
   float thr = -INFINITY;
-  for (int c = 0; c < parts; ++c) {
-    const size_t q = ((size_t)row * parts + c) * KP;
-    float f = -INFINITY;
-    int id = INVALID_ID;
-    if (lane < kout) {
-      f = __ldcg(sg.part_val + q + lane);
-      id = __ldcg(sg.part_id + q + lane);
+  for (int c0 = 0; c0 < parts; c0 += MERGE_BATCH) {
+    float f[MERGE_BATCH];
+    int id[MERGE_BATCH];
+#pragma unroll
+    for (int u = 0; u < MERGE_BATCH; ++u) {
+      f[u] = -INFINITY;
+      id[u] = INVALID_ID;
+      if (c0 + u < parts && lane < kout) {
+        const size_t q = ((size_t)row * parts + c0 + u) * KP;
+        f[u] = __ldcg(sg.part_val + q + lane);
+        id[u] = __ldcg(sg.part_id + q + lane);
+      }
     }
-    offer_scalars(f, id, thr, wv, wi, kout);
+#pragma unroll
+    for (int u = 0; u < MERGE_BATCH; ++u) offer_scalars(f[u], id[u], thr, wv, wi, kout);
   }
   float mm = -INFINITY, ss = 0.f;
   for (int c = lane; c < parts; c += 32) {
