@@ -203,7 +203,10 @@ brisk_status brisk_verify_block(const brisk_dims *dims, const void *logits_p,
  * hidden-state products; the proposal sweep, corrector and verification (the critical path);
  * the verifier-row sweep, which starts at once and fills the SMs the others leave free. When the
  * batch is small enough that the proposal rows are swept in several chunks each, the critical
- * path runs on `stream` itself and the verifier sweep starts after the proposal sweep. The call
+ * path runs on `stream` itself: the verifier sweep starts after the proposal sweep, beside the
+ * corrector; or, when both logit tensors together hold at most 64 MB, one sweep launch covers
+ * the rows of both and the corrector kernel also verifies (brisk_kernels_per_tail counts the
+ * launches). The call
  * only enqueues work and the results are ordered on `stream` (the side streams fork from and
  * join back to it, also under graph capture). The first call in a CUDA context creates the side
  * streams and their events: make it before any stream capture. Calls from several host threads

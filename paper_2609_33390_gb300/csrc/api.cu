@@ -30,10 +30,18 @@ bool dims_ok(const brisk_dims* d) {
 inline size_t esize(int dt) { return dt == BRISK_DT_BF16 ? 2 : 4; }
 
 // ---------------------------------------------------------------- workspace layout
+enum TailSchedule { SCHEDULE_OVERLAP = 0, SCHEDULE_SEPARATE = 1, SCHEDULE_FUSED = 2 };
+// Largest pair of logit tensors (bytes) for the fused small-batch schedule. Measured per block
+// (direct calls / graph replays): one sequence (16 MB) 124.9 / 106.4 us separate, 117.7 / 102.5
+// us fused; 16 sequences (259 MB, stochastic) 188.9 / 175.2 us separate, 243.6 / 210.6 fused.
+constexpr size_t FUSE_MAX_BYTES = size_t(64) << 20;
+
 struct WsLayout {
   size_t status, counters, part_val, part_id, part_m, part_s, argmax_p, lse_p;
   size_t cand_ids, cand_logprob, lse_q, sel, refined, Hm, G, G0, distill, base_rank, total;
-  int nchunk_q, nchunk_p, KP;   // chunks per proposal row (row layout) and verifier row (split)
+  int nchunk_q, nchunk_p, KP;   // chunks per proposal row (row layout) and verifier row
+  int mode_p;                   // layout of the verifier rows' sweep (SweepMode)
+  int schedule;                 // TailSchedule of brisk_decode_tail
 };
 
 WsLayout ws_layout(const brisk_dims* d) {
@@ -41,7 +49,21 @@ WsLayout ws_layout(const brisk_dims* d) {
   const size_t BL = (size_t)d->B * d->L;
   const size_t S = 2 * (size_t)d->r;
   w.nchunk_q = sweep_chunks((int)BL, d->V, d->logits_dtype, SWEEP_ROWS);
-  w.nchunk_p = sweep_chunks((int)BL, d->V, d->logits_dtype, SWEEP_SPLIT);
+  // Schedule of the fused tail and the verifier rows' layout (every entry point sweeps the
+  // verifier rows the same way, so that the fused and separate calls give the same bits):
+  //  OVERLAP  one task per proposal row: verifier rows in the split layout, beside the corrector;
+  //  FUSED    chunked proposal rows and both logit tensors within FUSE_MAX_BYTES: verifier rows
+  //           in the row layout with the proposal rows' chunks, both tensors in one launch;
+  //  SEPARATE chunked proposal rows, larger tensors: verifier rows in the split layout, beside
+  //           the corrector (the verifier sweep then takes long enough that overlapping it with
+  //           the corrector beats one launch before it).
+  const size_t sweep_bytes = 2 * BL * (size_t)d->V * esize(d->logits_dtype);
+  if (w.nchunk_q == 1) w.schedule = SCHEDULE_OVERLAP;
+  else w.schedule = sweep_bytes <= FUSE_MAX_BYTES ? SCHEDULE_FUSED : SCHEDULE_SEPARATE;
+  w.mode_p = w.schedule == SCHEDULE_FUSED ? SWEEP_ROWS : SWEEP_SPLIT;
+  w.nchunk_p = w.schedule == SCHEDULE_FUSED
+                   ? w.nchunk_q
+                   : sweep_chunks((int)BL, d->V, d->logits_dtype, SWEEP_SPLIT);
   w.KP = kp_for(d->K);
   const size_t np = BL * (size_t)(w.nchunk_q + w.nchunk_p);
   size_t o = 0;
@@ -446,7 +468,7 @@ brisk_status brisk_verify_block(const brisk_dims* d, const void* logits_p, const
                        at<float>(ws, w.lse_p));
   sw.nseg = 1;
   sw.V = d->V;
-  sw.mode = SWEEP_SPLIT;
+  sw.mode = w.mode_p;
   sw.nchunk = w.nchunk_p;
   sw.KP = w.KP;
   sw.dtype = d->logits_dtype;
@@ -520,18 +542,21 @@ brisk_status brisk::decode_tail_locked(const brisk_dims* d, const brisk_params* 
   // at once but only fills room the other two leave: the proposal sweep's ragged end (one
   // long task per row, ending over tens of microseconds) and the SMs beside the corrector.
   // In this mode the products use wide tiles (fewer SMs held at the start).
-  // With chunked proposal rows (few rows) the short tasks end together: then the critical path
-  // stays on A and the verifier sweep starts after the proposal sweep, beside the corrector,
-  // which saves the extra fork and keeps the SMs free for the corrector's start; the products,
-  // on the critical path there, use narrow tiles (more CTAs).
-  const bool overlap = w.nchunk_q == 1;
+  // With chunked proposal rows (few rows) the short tasks end together and the critical path
+  // stays on A, the products (on the critical path there) using narrow tiles (more CTAs):
+  //  SEPARATE the verifier sweep starts after the proposal sweep, beside the corrector, which
+  //           saves the extra fork and keeps the SMs free for the corrector's start;
+  //  FUSED    (small tensors) one sweep launch on A covers the rows of both tensors, and the
+  //           corrector that follows it verifies its sequence in the same CTA (four launches
+  //           with two products, against six).
+  const bool overlap = w.schedule == SCHEDULE_OVERLAP;
   SideStream* ss = side_stream();
   if (!ss) return BRISK_ERR_CUDA;
   cudaStream_t m = overlap ? ss->mid : st;
   BRISK_CUDA(cudaEventRecord(ss->ev[0], st));
   BRISK_CUDA(cudaStreamWaitEvent(ss->hi, ss->ev[0], 0));
   if (overlap) BRISK_CUDA(cudaStreamWaitEvent(m, ss->ev[0], 0));
-  BRISK_CUDA(cudaStreamWaitEvent(ss->lo, ss->ev[0], 0));
+  if (w.schedule != SCHEDULE_FUSED) BRISK_CUDA(cudaStreamWaitEvent(ss->lo, ss->ev[0], 0));
   s = hidden_products(d, p, tables, io->hidden, io->h_ctx, w, ws, ss->hi, overlap);
   if (s != BRISK_OK) return s;
   BRISK_CUDA(cudaEventRecord(ss->ev[1], ss->hi));
@@ -548,24 +573,8 @@ brisk_status brisk::decode_tail_locked(const brisk_dims* d, const brisk_params* 
   SweepLaunch sp = sq;
   sp.seg[0] = make_seg(w, ws, 1, io->logits_p, BL, 1, at<int32_t>(ws, w.argmax_p), nullptr,
                        at<float>(ws, w.lse_p));
-  sp.mode = SWEEP_SPLIT;
+  sp.mode = w.mode_p;
   sp.nchunk = w.nchunk_p;
-  if (ev && ev->sweep_q_begin) BRISK_CUDA(cudaEventRecord(static_cast<cudaEvent_t>(ev->sweep_q_begin), m));
-  BRISK_CUDA(launch_sweep(sq, m));
-  if (ev && ev->sweep_q_end) BRISK_CUDA(cudaEventRecord(static_cast<cudaEvent_t>(ev->sweep_q_end), m));
-  if (!overlap) {
-    BRISK_CUDA(cudaEventRecord(ss->ev[2], m));
-    BRISK_CUDA(cudaStreamWaitEvent(ss->lo, ss->ev[2], 0));
-  }
-
-  // verifier rows on the low-priority stream
-  if (ev && ev->sweep_p_begin) BRISK_CUDA(cudaEventRecord(static_cast<cudaEvent_t>(ev->sweep_p_begin), ss->lo));
-  BRISK_CUDA(launch_sweep(sp, ss->lo));
-  if (ev && ev->sweep_p_end) BRISK_CUDA(cudaEventRecord(static_cast<cudaEvent_t>(ev->sweep_p_end), ss->lo));
-  BRISK_CUDA(cudaEventRecord(ss->ev[3], ss->lo));
-
-  // the corrector once the proposal candidates and the hidden products are done
-  BRISK_CUDA(cudaStreamWaitEvent(m, ss->ev[1], 0));
   ScanArgs a = scan_args(d, p, tables, w, ws);
   a.select_mode = select_mode;
   a.verify_mode = verify_mode;
@@ -578,6 +587,48 @@ brisk_status brisk::decode_tail_locked(const brisk_dims* d, const brisk_params* 
   a.u_sel = io->u_sel;
   a.sel_tokens = sel;
   a.refined = refined;
+
+  if (w.schedule == SCHEDULE_FUSED) {
+    // both tensors' rows in one launch (the same layout and chunks as the separate calls)
+    SweepLaunch both = sq;
+    both.seg[1] = sp.seg[0];
+    both.nseg = 2;
+    if (ev && ev->sweep_q_begin) BRISK_CUDA(cudaEventRecord(static_cast<cudaEvent_t>(ev->sweep_q_begin), st));
+    if (ev && ev->sweep_p_begin) BRISK_CUDA(cudaEventRecord(static_cast<cudaEvent_t>(ev->sweep_p_begin), st));
+    BRISK_CUDA(launch_sweep(both, st));
+    if (ev && ev->sweep_q_end) BRISK_CUDA(cudaEventRecord(static_cast<cudaEvent_t>(ev->sweep_q_end), st));
+    if (ev && ev->sweep_p_end) BRISK_CUDA(cudaEventRecord(static_cast<cudaEvent_t>(ev->sweep_p_end), st));
+    // the corrector once the hidden products are done, verifying in the same CTA
+    BRISK_CUDA(cudaStreamWaitEvent(st, ss->ev[1], 0));
+    a.do_verify = 1;
+    a.logits_p = io->logits_p;
+    a.u_acc = io->u_acc;
+    a.u_res = io->u_res;
+    a.accepted_len = io->accepted_len;
+    a.out_tokens = io->out_tokens;
+    a.correction = io->correction;
+    a.next_anchor = io->next_anchor;
+    BRISK_CUDA(launch_scan(a, st));
+    return BRISK_OK;
+  }
+
+  if (ev && ev->sweep_q_begin) BRISK_CUDA(cudaEventRecord(static_cast<cudaEvent_t>(ev->sweep_q_begin), m));
+  BRISK_CUDA(launch_sweep(sq, m));
+  if (ev && ev->sweep_q_end) BRISK_CUDA(cudaEventRecord(static_cast<cudaEvent_t>(ev->sweep_q_end), m));
+  if (!overlap) {
+    // SEPARATE: the verifier rows after the proposal rows, beside the corrector
+    BRISK_CUDA(cudaEventRecord(ss->ev[2], m));
+    BRISK_CUDA(cudaStreamWaitEvent(ss->lo, ss->ev[2], 0));
+  }
+
+  // verifier rows on the low-priority stream
+  if (ev && ev->sweep_p_begin) BRISK_CUDA(cudaEventRecord(static_cast<cudaEvent_t>(ev->sweep_p_begin), ss->lo));
+  BRISK_CUDA(launch_sweep(sp, ss->lo));
+  if (ev && ev->sweep_p_end) BRISK_CUDA(cudaEventRecord(static_cast<cudaEvent_t>(ev->sweep_p_end), ss->lo));
+  BRISK_CUDA(cudaEventRecord(ss->ev[3], ss->lo));
+
+  // the corrector once the proposal candidates and the hidden products are done
+  BRISK_CUDA(cudaStreamWaitEvent(m, ss->ev[1], 0));
   BRISK_CUDA(launch_scan(a, m));
   BRISK_CUDA(cudaStreamWaitEvent(m, ss->ev[3], 0));
 
@@ -609,8 +660,11 @@ extern "C" {
 int32_t brisk_kernels_per_tail(const brisk_dims* dims) {
   if (!dims_ok(dims)) return 0;
   const bool tc = dims->hidden_dtype == BRISK_DT_BF16;
-  // two sweeps, the hidden-state products, the corrector scan, the verification
-  return 2 + (tc ? 2 : 4) + 1 + 1;
+  const int products = tc ? 2 : 4;
+  // two sweeps, the products, the corrector, the verification; in the fused small-batch
+  // schedule one sweep of both tensors, the products, the corrector that also verifies
+  if (ws_layout(dims).schedule != SCHEDULE_FUSED) return 2 + products + 1 + 1;
+  return 1 + products + 1;
 }
 
 brisk_status brisk_last_device_status(void* ws, int32_t clear, void* stream) {
@@ -693,7 +747,7 @@ brisk_status brisk_replay_diagnostics(const brisk_dims* d, const brisk_params* p
   SweepLaunch sp = sq;
   sp.seg[0] = make_seg(w, ws, 1, logits_p, BL, 1, at<int32_t>(ws, w.argmax_p), nullptr,
                        at<float>(ws, w.lse_p));
-  sp.mode = SWEEP_SPLIT;
+  sp.mode = w.mode_p;
   sp.nchunk = w.nchunk_p;
   BRISK_CUDA(launch_sweep(sp, st));
   // the head along the factual base prefix

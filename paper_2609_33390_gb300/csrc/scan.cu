@@ -418,10 +418,11 @@ struct CorrSmem {
   float* lprev;  // [L][K]  l_i(c_{i-1,k}); row 0 holds l_0(x0) in slot 0
   float* red;    // [2][NW][32] per-warp reduced residual dots (NW > 1)
   float* gpart;  // [2][NW]
+  Smem v;        // selections, ranks and refined scores kept for verification in the same CTA
 };
 
-__host__ __device__ inline size_t corr_layout(int L, int K, int S, int NW, char* base,
-                                              CorrSmem* sm) {
+__host__ __device__ inline size_t corr_layout(int L, int K, int S, int NW, int V, bool verify,
+                                              char* base, CorrSmem* sm) {
   size_t off = 0;
   auto take = [&](size_t bytes) {
     const size_t o = off;
@@ -436,10 +437,19 @@ __host__ __device__ inline size_t corr_layout(int L, int K, int S, int NW, char*
   char* pp = take(sizeof(float) * L * K);
   char* pr = take(sizeof(float) * 2 * NW * 32);
   char* pg = take(sizeof(float) * 2 * NW);
+  const size_t voff = off;
   if (sm) {
     sm->F = (float*)pF; sm->wg = (float*)pw;
     sm->cid = (int*)pc; sm->clp = (float*)pl; sm->top = (float*)pt; sm->lprev = (float*)pp;
     sm->red = (float*)pr; sm->gpart = (float*)pg;
+  }
+  // with verification in the same CTA its tables follow (the candidate table is the corrector's)
+  if (!verify) return off;
+  Smem v;
+  off = voff + smem_layout(L, K, S, V, base ? base + voff : nullptr, sm ? &v : nullptr);
+  if (sm) {
+    sm->v = v;
+    sm->v.cid = sm->cid;
   }
   return off;
 }
@@ -510,12 +520,16 @@ __device__ __forceinline__ void gather_logits(const void* logits, int dt, int n,
 // range, the surplus contributions multiplied by zero state or never read) so the compiler can
 // keep them all in flight. Candidate rows are read through L2, prefetched two positions ahead;
 // shared memory holds only small per-sequence tables.
-template <int NW, int NP, int CMC>
+// VERIFY: the CTA also verifies its sequence after the scan (the fused small-batch schedule); a
+// separate instantiation, since the verification code raises the scan's register count (168 ->
+// 228 a thread for four warps and K = 8), which would leave less room for the verifier-row
+// sweep beside the corrector in the overlapping schedule.
+template <int NW, int NP, int CMC, bool VERIFY>
 __global__ void __launch_bounds__(NW * 32)
 corrector_kernel(const __grid_constant__ ScanArgs a) {
   extern __shared__ __align__(16) char smem_raw[];
   CorrSmem sm;
-  corr_layout(a.L, a.K, a.S, NW, smem_raw, &sm);
+  corr_layout(a.L, a.K, a.S, NW, a.V, VERIFY, smem_raw, &sm);
   constexpr int NT = NW * 32;
   constexpr int LSTEP = 32 / NP;           // lane stride between reduced dots
   const int b = blockIdx.x;
@@ -753,7 +767,15 @@ corrector_kernel(const __grid_constant__ ScanArgs a) {
         set_status(a.status, BRISK_ERR_NUMERIC);
     }
     if (a.select_mode == BRISK_SELECT_SAMPLE && i + 1 < L) u_cur = a.u_sel[bL + i + 1];
-    if (tid == 0) a.sel_tokens[bL + i] = ci[pick];
+    if (tid == 0) {
+      a.sel_tokens[bL + i] = ci[pick];
+      if constexpr (VERIFY) {
+        sm.v.sel[i] = ci[pick];
+        sm.v.rank[i] = pick;
+      }
+    }
+    if constexpr (VERIFY)
+      if (warp == 0 && lane < K) sm.v.ref[i * K + lane] = ref;
     // the token fed forward: the head's selection, or in a same-state replay the base
     // selection (the Select rule on the base scores log q, same draw)
     int fwd = pick;
@@ -779,6 +801,12 @@ corrector_kernel(const __grid_constant__ ScanArgs a) {
       ts_id = ci[0];
     }
   }
+  // verification of this sequence in the same CTA (the verifier rows' statistics are complete:
+  // their sweep ran before this kernel)
+  if constexpr (VERIFY) {
+    __syncthreads();
+    verify_sequence(a, sm.v, b);
+  }
 }
 
 }  // namespace
@@ -787,18 +815,25 @@ size_t scan_smem_bytes(int L, int K, int S, int V) {
   return smem_layout(L, K, S, V, nullptr, nullptr);
 }
 
-template <int NP, int CMC, int NW = CORR_WARPS>
-cudaError_t launch_corrector(const ScanArgs& a, cudaStream_t stream) {
-  const size_t smem = corr_layout(a.L, a.K, a.S, NW, nullptr, nullptr);
-  cudaError_t e = cudaFuncSetAttribute(corrector_kernel<NW, NP, CMC>,
+template <int NW, int NP, int CMC, bool VERIFY>
+cudaError_t launch_corrector_k(const ScanArgs& a, cudaStream_t stream) {
+  const size_t smem = corr_layout(a.L, a.K, a.S, NW, a.V, VERIFY, nullptr, nullptr);
+  cudaError_t e = cudaFuncSetAttribute(corrector_kernel<NW, NP, CMC, VERIFY>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  if (e == cudaSuccess) e = prefer_carveout(corrector_kernel<NW, NP, CMC>, CARVEOUT_SMALL_KB);
+  if (e == cudaSuccess) e = prefer_carveout(corrector_kernel<NW, NP, CMC, VERIFY>, CARVEOUT_SMALL_KB);
   if (e != cudaSuccess) return e;
-  corrector_kernel<NW, NP, CMC><<<a.B, NW * 32, smem, stream>>>(a);
+  corrector_kernel<NW, NP, CMC, VERIFY><<<a.B, NW * 32, smem, stream>>>(a);
   return cudaGetLastError();
 }
 
-// The corrector (do_select) or the verification (do_verify) for every sequence.
+template <int NP, int CMC, int NW = CORR_WARPS>
+cudaError_t launch_corrector(const ScanArgs& a, cudaStream_t stream) {
+  if (a.do_verify) return launch_corrector_k<NW, NP, CMC, true>(a, stream);
+  return launch_corrector_k<NW, NP, CMC, false>(a, stream);
+}
+
+// The corrector (do_select; with do_verify also the verification in the same CTA) or the
+// verification alone (do_verify) for every sequence.
 cudaError_t launch_scan(const ScanArgs& a, cudaStream_t stream) {
   if (a.do_select) {
     // 4-element chunks per lane: S / 4 chunks over the CTA's lanes. A state wider than four
