@@ -706,6 +706,10 @@ def run_profile(args):
     build.build()
     dev = torch.device("cuda")
     wl = synth.WORKLOADS[args.profile]
+    if args.profile_batch:
+        wl = wl.with_(B=args.profile_batch)
+    if args.profile_vocab:
+        wl = wl.with_(V=args.profile_vocab)
     weights = synth.make_weights(wl, dev)
     tail = brisk.DecodeTail.for_workload(wl, weights, dev)
     tail.prepare()
@@ -716,7 +720,7 @@ def run_profile(args):
         tail.tail(blk, sm, vm, out=out)
     torch.cuda.synchronize()
     st = tail.device_status()
-    print(json.dumps({"profile": args.profile, "calls": args.warmup + args.steps,
+    print(json.dumps({"profile": args.profile, "B": wl.B, "V": wl.V, "calls": args.warmup + args.steps,
                       "status": brisk.status_string(st),
                       "accepted": int(out["accepted_len"].sum())}))
     return 0 if st == brisk.OK else 1
@@ -735,6 +739,10 @@ def main(argv=None):
                     help="skip the measurements of the other four workload configurations")
     ap.add_argument("--per-config-steps", type=int, default=20)
     ap.add_argument("--profile", default=None, help="workload name: short untimed run for ncu")
+    ap.add_argument("--profile-batch", type=int, default=0,
+                    help="with --profile: sequences per call instead of the workload's (a smaller case)")
+    ap.add_argument("--profile-vocab", type=int, default=0,
+                    help="with --profile: vocabulary size instead of the workload's (a smaller case)")
     args = ap.parse_args(argv)
     args.warmup = max(3, args.warmup)   # at least 3 untimed warm-up steps
     if args.profile:
