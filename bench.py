@@ -71,6 +71,21 @@ def measured_peaks():
     return FALLBACK_HBM_GBS, "fallback"
 
 
+def bf16_peak_tflops() -> float:
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            return float(json.load(f)["bf16_tflops"])
+    return 1900.0
+
+
+def fold_flops_of(wl) -> float:
+    """Algorithmic flops of the once-per-weight-set folds: P_e E_in(v) and W_c E_out(v) (k = d),
+    the token shares of the gate, candidate and Init pre-activations (2S + S outputs, k = r) and
+    the residual rows (S outputs, k = r), for every token v."""
+    return 2.0 * wl.V * wl.r * (2 * wl.d + 4 * wl.S)
+
+
 def sweep_source_hash() -> str:
     """Hash of the sweep source's code: line comments, trailing blanks and empty lines are left
     out, so that an edit of the comments alone keeps a traffic record that is still valid."""
@@ -327,10 +342,13 @@ def run_ours(args):
 
     weights = synth.make_weights(wl, dev)
     tail = brisk.DecodeTail.for_workload(wl, weights, dev)
+    tail.prepare()               # the first call sets kernel attributes; time the second
+    torch.cuda.synchronize()
     t = time.perf_counter()
     tail.prepare()
     torch.cuda.synchronize()
     prepare_ms = 1000.0 * (time.perf_counter() - t)
+    fold_flops = fold_flops_of(wl)
 
     pool_n = max(1, min(args.pool, args.steps + args.warmup))
     pool = []
@@ -487,7 +505,10 @@ def run_ours(args):
         "config": {**workload_config(wl),
                    "l2": f"inputs larger than L2 ({sweep_bytes / 1e9:.2f} GB of logits per step,"
                          f" {pool_n} distinct blocks cycled)",
-                   "prepare_ms": round(prepare_ms, 1)},
+                   "prepare_ms": round(prepare_ms, 1),
+                   "prepare_tflops": round(fold_flops / (prepare_ms * 1e-3) / 1e12, 1),
+                   "prepare_frac_of_bf16_peak": round(fold_flops / (prepare_ms * 1e-3) / 1e12
+                                                      / bf16_peak_tflops(), 3)},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "traffic": traffic, "peak_source": peak_src,
                      "kernel": "sweep_kernel (proposal rows + verifier rows, two overlapping "

@@ -95,14 +95,15 @@ WsLayout ws_layout(const brisk_dims* d) {
 //              Tz(v) = W_z[:, r:2r] P_e E_in(v), Th(v) = W_h[:, r:2r] P_e E_in(v)
 // U   [V, S] : residual rows, U(v) = W_s^T W_c E_out(v)
 // T0  [V, S] : token share of Init, W0[:, r:2r] P_e E_in(v)
-// Tin, Tout [V, r]: P_e E_in(v), W_c E_out(v) (intermediates of the folds)
+// Tin, Tout [V, r]: P_e E_in(v), W_c E_out(v) (intermediates of the folds; on the tensor-core
+//              path their space holds one of them at a time as three bf16 parts [V, 3r])
 // posG [L, 2S]: position shares W_z[:, 2r:2r+16] pos_i | W_h[:, 2r:2r+16] pos_i
 // Fz, Fh [S, 5]: feature shares W_z[:, 2r+16:] P_phi, W_h[:, 2r+16:] P_phi
 // wg [S+5] fp32 copy of w_g; W2 [2S, r] = [W_z[:, :r] ; W_h[:, :r]] and W0h [S, r] = W0[:, :r] (fp32)
 // W2s [2S, 3r], W0s [S, 3r] (bf16): the same blocks written three times along k, so that
 // [hi | mid | lo] W^T = (hi + mid + lo) W^T on bf16 tensor cores.
 struct TbLayout {
-  size_t Tzh, U, T0, Tin, Tout, posG, Fz, Fh, wg, W2, W0h, W2s, W0s, total;
+  size_t Tzh, U, T0, Tin, Tout, posG, Fz, Fh, wg, W2, W0h, W2s, W0s, Wt2s, W0ts, Ws3, total;
 };
 
 TbLayout tb_layout(const brisk_dims* d) {
@@ -123,6 +124,11 @@ TbLayout tb_layout(const brisk_dims* d) {
   t.W0h = take(sizeof(float) * S * r);
   t.W2s = take(2 * 2 * S * 3 * r);
   t.W0s = take(2 * S * 3 * r);
+  // bf16 token-side blocks written three times along k, for the folds on the tensor cores:
+  // [W_z[:, r:2r] ; W_h[:, r:2r]] [2S, 3r], W0[:, r:2r] [S, 3r], W_s^T [S, 3r]
+  t.Wt2s = take(2 * 2 * S * 3 * r);
+  t.W0ts = take(2 * S * 3 * r);
+  t.Ws3 = take(2 * S * 3 * r);
   t.total = o;
   return t;
 }
@@ -351,16 +357,42 @@ brisk_status brisk_corrector_prepare(const brisk_dims* d, const brisk_params* p,
   float* Tin = at<float>(tables, t.Tin);
   float* Tout = at<float>(tables, t.Tout);
   float* Tzh = at<float>(tables, t.Tzh);
-  // P_e E_in(v) and W_c E_out(v) for every v
-  BRISK_CUDA(gemm_simt(V, r, d->d, p->E_in, hd, d->d, p->P_e, hd, d->d, false, Tin, r, st));
-  BRISK_CUDA(gemm_simt(V, r, d->d, p->E_out, hd, d->d, p->W_c, hd, d->d, false, Tout, r, st));
-  // token shares of the gate / candidate pre-activations and of Init
-  BRISK_CUDA(gemm_simt(V, S, r, Tin, F32, r, wp(p->Wz, r), hd, ldw, false, Tzh, 2 * S, st));
-  BRISK_CUDA(gemm_simt(V, S, r, Tin, F32, r, wp(p->Wh, r), hd, ldw, false, Tzh + S, 2 * S, st));
-  BRISK_CUDA(gemm_simt(V, S, r, Tin, F32, r, wp(p->W0, r), hd, 2 * r, false, at<float>(tables, t.T0),
-                       S, st));
-  // residual rows U(v) = W_s^T (W_c E_out(v)): B(n=j, k=t) = W_s[t, j]
-  BRISK_CUDA(gemm_simt(V, S, r, Tout, F32, r, p->W_s, hd, S, true, at<float>(tables, t.U), S, st));
+  if (hd == BRISK_DT_BF16 && gemm_tc_supported(p->E_in, d->d, p->P_e, d->d, d->d) &&
+      gemm_tc_supported(p->E_out, d->d, p->W_c, d->d, d->d)) {
+    // On the tensor cores. P_e E_in(v) (then W_c E_out(v)) is written as three bf16 parts
+    // (hi + mid + lo, exact to about 2^-24 relative) into the Tin / Tout space, and the next
+    // products multiply the parts by the weight blocks written three times along k, which keeps
+    // fp32-level accuracy on bf16 tensor cores. No status word: a bounded wait that gives up
+    // here (about 2 s at the default limit) leaves the tables undefined.
+    const int BF = BRISK_DT_BF16, r3 = 3 * r;
+    __nv_bfloat16* Wt2s = at<__nv_bfloat16>(tables, t.Wt2s);
+    __nv_bfloat16* W0ts = at<__nv_bfloat16>(tables, t.W0ts);
+    __nv_bfloat16* Ws3 = at<__nv_bfloat16>(tables, t.Ws3);
+    for (int part = 0; part < 3; ++part) {
+      BRISK_CUDA(copy2d(S, r, wp(p->Wz, r), hd, ldw, Wt2s + part * r, BF, r3, st));
+      BRISK_CUDA(copy2d(S, r, wp(p->Wh, r), hd, ldw, Wt2s + (size_t)S * r3 + part * r, BF, r3, st));
+      BRISK_CUDA(copy2d(S, r, wp(p->W0, r), hd, 2 * r, W0ts + part * r, BF, r3, st));
+      BRISK_CUDA(copy2d(S, r, p->W_s, hd, S, Ws3 + part * r, BF, r3, st, true));   // W_s^T
+    }
+    __nv_bfloat16* X3 = at<__nv_bfloat16>(tables, t.Tin);   // [V, 3r] in the Tin and Tout space
+    BRISK_CUDA(gemm_tc(V, r, d->d, p->E_in, d->d, p->P_e, d->d, 1, X3, r3, nullptr, st));
+    const TcSpec tok[2] = {{V, 2 * S, r3, X3, r3, Wt2s, r3, 0, Tzh, 2 * S, nullptr, 0, 0},
+                           {V, S, r3, X3, r3, W0ts, r3, 0, at<float>(tables, t.T0), S, nullptr, 0, 0}};
+    BRISK_CUDA(gemm_tc_grouped(tok, 2, nullptr, st, 4));
+    BRISK_CUDA(gemm_tc(V, r, d->d, p->E_out, d->d, p->W_c, d->d, 1, X3, r3, nullptr, st));
+    BRISK_CUDA(gemm_tc(V, S, r3, X3, r3, Ws3, r3, 0, at<float>(tables, t.U), S, nullptr, st));
+  } else {
+    // P_e E_in(v) and W_c E_out(v) for every v
+    BRISK_CUDA(gemm_simt(V, r, d->d, p->E_in, hd, d->d, p->P_e, hd, d->d, false, Tin, r, st));
+    BRISK_CUDA(gemm_simt(V, r, d->d, p->E_out, hd, d->d, p->W_c, hd, d->d, false, Tout, r, st));
+    // token shares of the gate / candidate pre-activations and of Init
+    BRISK_CUDA(gemm_simt(V, S, r, Tin, F32, r, wp(p->Wz, r), hd, ldw, false, Tzh, 2 * S, st));
+    BRISK_CUDA(gemm_simt(V, S, r, Tin, F32, r, wp(p->Wh, r), hd, ldw, false, Tzh + S, 2 * S, st));
+    BRISK_CUDA(gemm_simt(V, S, r, Tin, F32, r, wp(p->W0, r), hd, 2 * r, false,
+                         at<float>(tables, t.T0), S, st));
+    // residual rows U(v) = W_s^T (W_c E_out(v)): B(n=j, k=t) = W_s[t, j]
+    BRISK_CUDA(gemm_simt(V, S, r, Tout, F32, r, p->W_s, hd, S, true, at<float>(tables, t.U), S, st));
+  }
   // position shares
   BRISK_CUDA(gemm_simt(L, S, 16, p->pos, hd, 16, wp(p->Wz, 2 * r), hd, ldw, false,
                        at<float>(tables, t.posG), 2 * S, st));

@@ -303,9 +303,9 @@ struct TcSpec {
 cudaError_t gemm_tc_grouped(const TcSpec* spec, int nprob, int32_t* status, cudaStream_t stream,
                             int stages);
 bool gemm_tc_supported(const void* A, int lda, const void* B, int ldb, int K);
-// dst[i*ldd + j] = (dst type) src[i*lds + j], i < rows, j < cols.
+// dst[i*ldd + j] = (dst type) src[i*lds + j], i < rows, j < cols (src[j*lds + i] with transpose).
 cudaError_t copy2d(int rows, int cols, const void* src, int s_dt, int lds, void* dst, int d_dt,
-                   int ldd, cudaStream_t stream);
+                   int ldd, cudaStream_t stream, bool transpose = false);
 
 // ---------------------------------------------------------------- corrector scan and verify
 struct ScanArgs {

@@ -102,12 +102,12 @@ gemm_skinny_kernel(int M, int N, int K, const TA* __restrict__ A, int lda,
 
 template <typename TS, typename TD>
 __global__ void copy2d_kernel(int rows, int cols, const TS* __restrict__ src, int lds,
-                              TD* __restrict__ dst, int ldd) {
+                              TD* __restrict__ dst, int ldd, int transpose) {
   const long long n = (long long)rows * cols;
   for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < n;
        e += (long long)gridDim.x * blockDim.x) {
     const long long i = e / cols, j = e % cols;
-    const float v = to_f32(src[i * lds + j]);
+    const float v = to_f32(transpose ? src[j * lds + i] : src[i * lds + j]);
     if constexpr (sizeof(TD) == 4) dst[i * ldd + j] = v;
     else dst[i * ldd + j] = __float2bfloat16_rn(v);
   }
@@ -133,15 +133,16 @@ cudaError_t gemm_t(int M, int N, int K, const void* A, int lda, const void* B, i
 
 template <typename TS>
 cudaError_t copy_t(int rows, int cols, const void* src, int lds, void* dst, int d_dt, int ldd,
-                   cudaStream_t stream) {
+                   bool transpose, cudaStream_t stream) {
   const long long n = (long long)rows * cols;
   const unsigned grid = (unsigned)((n + 255) / 256 > 4096 ? 4096 : (n + 255) / 256);
   if (d_dt == BRISK_DT_F32)
     copy2d_kernel<TS, float><<<grid, 256, 0, stream>>>(rows, cols, static_cast<const TS*>(src), lds,
-                                                       static_cast<float*>(dst), ldd);
+                                                       static_cast<float*>(dst), ldd, transpose);
   else
     copy2d_kernel<TS, __nv_bfloat16><<<grid, 256, 0, stream>>>(
-        rows, cols, static_cast<const TS*>(src), lds, static_cast<__nv_bfloat16*>(dst), ldd);
+        rows, cols, static_cast<const TS*>(src), lds, static_cast<__nv_bfloat16*>(dst), ldd,
+        transpose);
   return cudaGetLastError();
 }
 
@@ -164,10 +165,11 @@ cudaError_t gemm_simt(int M, int N, int K, const void* A, int a_dt, int lda, con
 }
 
 cudaError_t copy2d(int rows, int cols, const void* src, int s_dt, int lds, void* dst, int d_dt,
-                   int ldd, cudaStream_t stream) {
+                   int ldd, cudaStream_t stream, bool transpose) {
   if (rows <= 0 || cols <= 0) return cudaSuccess;
-  if (s_dt == BRISK_DT_BF16) return copy_t<__nv_bfloat16>(rows, cols, src, lds, dst, d_dt, ldd, stream);
-  return copy_t<float>(rows, cols, src, lds, dst, d_dt, ldd, stream);
+  if (s_dt == BRISK_DT_BF16)
+    return copy_t<__nv_bfloat16>(rows, cols, src, lds, dst, d_dt, ldd, transpose, stream);
+  return copy_t<float>(rows, cols, src, lds, dst, d_dt, ldd, transpose, stream);
 }
 
 }  // namespace brisk
