@@ -201,8 +201,10 @@ brisk_status brisk_verify_block(const brisk_dims *dims, const void *logits_p,
  * results, bit for bit, as brisk_topk_candidates + brisk_corrector_select + brisk_verify_block on
  * the same inputs. The work runs on library side streams of decreasing priority: the
  * hidden-state products; the proposal sweep, corrector and verification (the critical path);
- * the verifier-row sweep, which starts at once and fills the SMs the others leave free. When the
- * batch is small enough that the proposal rows are swept in several chunks each, the critical
+ * the verifier-row sweep, which starts at once and fills the SMs the others leave free (this
+ * applies whenever each proposal row is swept as one task: many rows, or rows too short to
+ * split). When the batch is small enough that the proposal rows are swept in several chunks
+ * each, the critical
  * path runs on `stream` itself: the verifier sweep starts after the proposal sweep, beside the
  * corrector; or, when both logit tensors together hold at most 64 MB, one sweep launch covers
  * the rows of both and the corrector kernel also verifies (brisk_kernels_per_tail counts the

@@ -110,3 +110,22 @@ def test_wait_limit_setter_returns_the_previous_limit(B):
         assert B.set_wait_limit(99) == default
     finally:
         B.set_wait_limit(0)
+
+
+def test_kernels_per_tail_follows_the_schedule(B):
+    """Four launches in the fused small-batch schedule (one sweep of both tensors, two tensor-core
+    products, the corrector that verifies), six otherwise; four SIMT products with fp32 weights."""
+    fused = _dims(B, B=2, L=8, V=65536, d=64, K=8, r=16)          # chunked rows, 4 MB of logits
+    separate = _dims(B, B=4, L=32, V=140000, d=64, K=8, r=16)     # chunked rows, 72 MB
+    overlap = _dims(B, B=128, L=32, V=126464, d=4096, K=8, r=256)  # one task a row (many rows)
+    short_rows = _dims(B, B=2, L=8, V=4096, d=64, K=8, r=16)      # one task a row (rows too short)
+    assert B.kernels_per_tail(fused) == 4
+    assert B.kernels_per_tail(separate) == 6
+    assert B.kernels_per_tail(overlap) == 6
+    assert B.kernels_per_tail(short_rows) == 6
+    assert B.kernels_per_tail(_dims(B, B=2, L=8, V=65536, d=64, K=8, r=16,
+                                    hidden_dtype=torch.float32)) == 6
+    assert B.kernels_per_tail(_dims(B, B=2, L=8, V=4096, d=64, K=8, r=16,
+                                    hidden_dtype=torch.float32)) == 8
+    bad = _dims(B, K=3)
+    assert B.kernels_per_tail(bad) == 0

@@ -153,6 +153,38 @@ def test_overlap_schedule_matches_unfused(brisk):
     assert rep.sequences == 4
 
 
+def test_separate_schedule_matches_unfused(brisk):
+    """Chunked proposal rows with both logit tensors above 64 MB take the separate small-batch
+    schedule (the verifier sweep beside the corrector, six launches): bit for bit the same as
+    the three separate calls, and parity with the oracle."""
+    wl = synth.Workload("separate", B=4, L=32, V=140000, d=64, K=8, r=16, agree0=0.9,
+                        agree_decay=0.97, weight_std=0.2)
+    dims = brisk.make_dims(wl.B, wl.L, wl.V, wl.d, wl.K, wl.r, wl.logits_dtype, wl.hidden_dtype)
+    assert brisk.kernels_per_tail(dims) == 6
+    weights = _to(synth.make_weights(wl, "cpu"), "cuda")
+    block = _to(synth.make_block(wl, "cpu"), "cuda")
+    rep, g = _run_and_check(brisk, wl, weights, block, unfused=True)
+    assert rep.sequences == wl.B
+
+
+@pytest.mark.parametrize("modes", [("sample", "stochastic"), ("greedy", "stochastic"),
+                                   ("greedy", "greedy")])
+def test_fused_schedule_matches_unfused(brisk, modes):
+    """Chunked proposal rows with both logit tensors within 64 MB take the fused small-batch
+    schedule (one sweep of both tensors, the corrector verifying in the same CTA, four launches),
+    in every mode pair: bit for bit the same as the three separate calls, and parity with the
+    oracle."""
+    sm_, vm_ = modes
+    wl = synth.Workload("fused", B=3, L=8, V=65536, d=64, K=8, r=16, select_mode=sm_,
+                        verify_mode=vm_, agree0=0.8, agree_decay=0.9, weight_std=0.2)
+    dims = brisk.make_dims(wl.B, wl.L, wl.V, wl.d, wl.K, wl.r, wl.logits_dtype, wl.hidden_dtype)
+    assert brisk.kernels_per_tail(dims) == 4
+    weights = _to(synth.make_weights(wl, "cpu"), "cuda")
+    block = _to(synth.make_block(wl, "cpu"), "cuda")
+    rep, g = _run_and_check(brisk, wl, weights, block, unfused=True)
+    assert rep.sequences == wl.B
+
+
 def test_non_finite_row_sets_numeric_status(brisk):
     wl = synth.Workload("nan", B=1, L=3, V=512, d=16, K=4, r=16)
     weights = _to(synth.make_weights(wl, "cpu"), "cuda")
