@@ -233,6 +233,29 @@ __device__ __forceinline__ void mbar_drain(uint64_t* bar, uint32_t parity) {
 __device__ __forceinline__ void fence_async_smem() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
+// Launches `kernel` with the priority of `stream` as a launch attribute. Kernel nodes captured
+// into a CUDA graph keep launch attributes, but not the priority of the stream they were captured
+// from, so without it a replay of the tail's three-priority schedule runs every kernel at the
+// default priority.
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_prio(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                               cudaStream_t stream, Args&&... args) {
+  int prio = 0;
+  cudaError_t e = cudaStreamGetPriority(stream, &prio);
+  if (e != cudaSuccess) return e;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributePriority;
+  attr[0].val.priority = prio;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
+
 __device__ __forceinline__ void set_status(int32_t* status, int code) {
   if (status) atomicCAS(status, 0, code);
 }

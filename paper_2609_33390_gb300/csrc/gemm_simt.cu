@@ -119,16 +119,17 @@ cudaError_t gemm_t(int M, int N, int K, const void* A, int lda, const void* B, i
                    int bias_period) {
   if (M <= SKINNY_MAX_M && !transB) {
     const unsigned grid = (unsigned)((N + SKINNY_WARPS - 1) / SKINNY_WARPS);
-    gemm_skinny_kernel<TA, TB><<<grid, SKINNY_WARPS * 32, 0, stream>>>(
-        M, N, K, static_cast<const TA*>(A), lda, static_cast<const TB*>(B), ldb, C, ldc, bias,
+    const cudaError_t e = launch_prio(
+        gemm_skinny_kernel<TA, TB>, dim3(grid), dim3(SKINNY_WARPS * 32), 0, stream, M, N, K,
+        static_cast<const TA*>(A), lda, static_cast<const TB*>(B), ldb, C, ldc, bias,
         bias_period > 0 ? bias_period : 1);
-    return cudaGetLastError();
+    return e != cudaSuccess ? e : cudaGetLastError();
   }
   const dim3 grid((N + TN - 1) / TN, (M + TM - 1) / TM);
-  gemm_simt_kernel<TA, TB><<<grid, 256, 0, stream>>>(
+  const cudaError_t e = launch_prio(gemm_simt_kernel<TA, TB>, grid, dim3(256), 0, stream,
       M, N, K, static_cast<const TA*>(A), lda, static_cast<const TB*>(B), ldb, transB ? 1 : 0, C, ldc,
       bias, bias_period > 0 ? bias_period : 1);
-  return cudaGetLastError();
+  return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 template <typename TS>

@@ -465,7 +465,8 @@ cudaError_t gemm_tc_grouped(const TcSpec* spec, int nprob, int32_t* status, cuda
   if (e == cudaSuccess) e = stages == 2 ? prefer_carveout(gemm_tc_kernel<2>, CARVEOUT_GEMM_KB)
                                         : prefer_carveout(gemm_tc_kernel<4>, CARVEOUT_GEMM_KB);
   if (e != cudaSuccess) return e;
-  kernel<<<total, TC_THREADS, smem, stream>>>(maps, a);
+  e = launch_prio(kernel, dim3(total), dim3(TC_THREADS), smem, stream, maps, a);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 

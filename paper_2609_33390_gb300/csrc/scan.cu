@@ -822,7 +822,8 @@ cudaError_t launch_corrector_k(const ScanArgs& a, cudaStream_t stream) {
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e == cudaSuccess) e = prefer_carveout(corrector_kernel<NW, NP, CMC, VERIFY>, CARVEOUT_SMALL_KB);
   if (e != cudaSuccess) return e;
-  corrector_kernel<NW, NP, CMC, VERIFY><<<a.B, NW * 32, smem, stream>>>(a);
+  e = launch_prio(corrector_kernel<NW, NP, CMC, VERIFY>, dim3(a.B), dim3(NW * 32), smem, stream, a);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 
@@ -855,7 +856,8 @@ cudaError_t launch_scan(const ScanArgs& a, cudaStream_t stream) {
   if (e == cudaSuccess) e = prefer_carveout(verify_kernel, CARVEOUT_SMALL_KB);
   if (e != cudaSuccess) return e;
   const int threads = a.verify_mode == BRISK_VERIFY_STOCHASTIC ? VERIFY_THREADS_MAX : VERIFY_THREADS;
-  verify_kernel<<<a.B, threads, smem, stream>>>(a);
+  e = launch_prio(verify_kernel, dim3(a.B), dim3(threads), smem, stream, a);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 

@@ -456,14 +456,16 @@ cudaError_t launch_t(const SweepLaunch& a, cudaStream_t stream) {
   if (a.mode == SWEEP_ROWS) {
     const long long tasks = rows * a.nchunk;
     const unsigned grid = (unsigned)((tasks + SWEEP_ROW_WARPS - 1) / SWEEP_ROW_WARPS);
-    const cudaError_t e = prefer_carveout(sweep_kernel<T, SWEEP_ROWS>, CARVEOUT_SMALL_KB);
+    cudaError_t e = prefer_carveout(sweep_kernel<T, SWEEP_ROWS>, CARVEOUT_SMALL_KB);
     if (e != cudaSuccess) return e;
-    sweep_kernel<T, SWEEP_ROWS><<<grid, SWEEP_ROW_WARPS * 32, 0, stream>>>(a);
+    e = launch_prio(sweep_kernel<T, SWEEP_ROWS>, dim3(grid), dim3(SWEEP_ROW_WARPS * 32), 0, stream, a);
+    if (e != cudaSuccess) return e;
   } else {
     const unsigned grid = (unsigned)(rows * (a.nchunk / SWEEP_WARPS));
-    const cudaError_t e = prefer_carveout(sweep_kernel<T, SWEEP_SPLIT>, CARVEOUT_SMALL_KB);
+    cudaError_t e = prefer_carveout(sweep_kernel<T, SWEEP_SPLIT>, CARVEOUT_SMALL_KB);
     if (e != cudaSuccess) return e;
-    sweep_kernel<T, SWEEP_SPLIT><<<grid, SWEEP_WARPS * 32, 0, stream>>>(a);
+    e = launch_prio(sweep_kernel<T, SWEEP_SPLIT>, dim3(grid), dim3(SWEEP_WARPS * 32), 0, stream, a);
+    if (e != cudaSuccess) return e;
   }
   return cudaGetLastError();
 }
