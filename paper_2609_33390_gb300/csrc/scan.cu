@@ -74,6 +74,42 @@ __device__ __forceinline__ float4 add4(float4 x, float4 y) {
 __device__ __forceinline__ float4 ldcg4(const float* p) {
   return __ldcg(reinterpret_cast<const float4*>(p));
 }
+
+// A lane's chunk of CW consecutive state elements (CW = 2 or 4), loaded as one vector.
+template <int CW>
+struct Chunk {
+  float v[CW];
+};
+template <int CW>
+__device__ __forceinline__ Chunk<CW> chunk_of(const float4& t) {
+  if constexpr (CW == 4) return {{t.x, t.y, t.z, t.w}};
+  else return {{t.x, t.y}};
+}
+template <int CW, bool CG>
+__device__ __forceinline__ Chunk<CW> ldc(const float* p) {
+  if constexpr (CW == 4) {
+    return chunk_of<4>(CG ? __ldcg(reinterpret_cast<const float4*>(p))
+                          : *reinterpret_cast<const float4*>(p));
+  } else {
+    const float2 t = CG ? __ldcg(reinterpret_cast<const float2*>(p))
+                        : *reinterpret_cast<const float2*>(p);
+    return {{t.x, t.y}};
+  }
+}
+template <int CW>
+__device__ __forceinline__ Chunk<CW> addc(const Chunk<CW>& x, const Chunk<CW>& y) {
+  Chunk<CW> r;
+#pragma unroll
+  for (int e = 0; e < CW; ++e) r.v[e] = x.v[e] + y.v[e];
+  return r;
+}
+// acc + sum_e x_e y_e, the last element first (the order of the four-element form)
+template <int CW>
+__device__ __forceinline__ float dotc(const Chunk<CW>& x, const Chunk<CW>& y, float acc) {
+#pragma unroll
+  for (int e = CW - 1; e >= 0; --e) acc = fmaf(x.v[e], y.v[e], acc);
+  return acc;
+}
 // Logistic function with the hardware exponential (relative error ~1e-6).
 __device__ __forceinline__ float sigmoid_fast(float x) { return __fdividef(1.f, 1.f + __expf(-x)); }
 
@@ -510,7 +546,7 @@ __device__ __forceinline__ void gather_logits(const void* logits, int dt, int n,
 }
 
 // The sequential corrector (Sec. 3.3 Eqs. 4-5; App. C.3 Eq. 9; Algorithm 1(b) loop), one CTA of
-// NW warps per sequence. Lane l of warp w owns the 4-element state chunks
+// NW warps per sequence. Lane l of warp w owns the CW-element state chunks (CW = 2 or 4)
 // c = l + 32 (w + NW m), m < CMC. The residual dots and the gate are reduced with warp
 // shuffles, then across the warps through shared memory (one block barrier a position), and
 // Select runs in every warp with lane k holding candidate k. Spreading a sequence over the
@@ -524,7 +560,7 @@ __device__ __forceinline__ void gather_logits(const void* logits, int dt, int n,
 // separate instantiation, since the verification code raises the scan's register count (168 ->
 // 228 a thread for four warps and K = 8), which would leave less room for the verifier-row
 // sweep beside the corrector in the overlapping schedule.
-template <int NW, int NP, int CMC, bool VERIFY>
+template <int NW, int NP, int CMC, int CW, bool VERIFY>
 __global__ void __launch_bounds__(NW * 32)
 corrector_kernel(const __grid_constant__ ScanArgs a) {
   extern __shared__ __align__(16) char smem_raw[];
@@ -536,7 +572,7 @@ corrector_kernel(const __grid_constant__ ScanArgs a) {
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int L = a.L, K = a.K, S = a.S, V = a.V;
   const size_t bL = (size_t)b * L;
-  const int nch = S / 4;
+  const int nch = S / CW;
 
   for (int e = tid; e < L * K; e += NT) {
     int c = a.cand_ids[bL * K + e];
@@ -583,18 +619,20 @@ corrector_kernel(const __grid_constant__ ScanArgs a) {
     ok[m] = c < nch;
     cc[m] = ok[m] ? c : nch - 1;
   }
-  float4 s4[CMC], gz4[CMC], gh4[CMC], tz4[CMC], th4[CMC];
+  using C = Chunk<CW>;
+  C s4[CMC], gz4[CMC], gh4[CMC], tz4[CMC], th4[CMC];
 #pragma unroll
   for (int m = 0; m < CMC; ++m) {
     const int c = cc[m];
-    const float4 g0 = ldcg4(a.G0 + (size_t)b * S + 4 * c), t0 = ldcg4(a.T0 + (size_t)x0 * S + 4 * c);
-    s4[m] = ok[m] ? make_float4(tanhf(g0.x + t0.x), tanhf(g0.y + t0.y), tanhf(g0.z + t0.z),
-                                tanhf(g0.w + t0.w))        // s_{-1} = u_0 = Init(h_c, E(x0))
-                  : make_float4(0.f, 0.f, 0.f, 0.f);
-    gz4[m] = add4(ldcg4(a.G + bL * 2 * S + 4 * c), ld4(a.posG + 4 * c));
-    gh4[m] = add4(ldcg4(a.G + bL * 2 * S + S + 4 * c), ld4(a.posG + S + 4 * c));
-    tz4[m] = ldcg4(a.Tzh + (size_t)x0 * 2 * S + 4 * c);   // token share of x_{-1} = x0
-    th4[m] = ldcg4(a.Tzh + (size_t)x0 * 2 * S + S + 4 * c);
+    const C g0 = ldc<CW, true>(a.G0 + (size_t)b * S + CW * c);
+    const C t0 = ldc<CW, true>(a.T0 + (size_t)x0 * S + CW * c);
+#pragma unroll
+    for (int e = 0; e < CW; ++e)                              // s_{-1} = u_0 = Init(h_c, E(x0))
+      s4[m].v[e] = ok[m] ? tanhf(g0.v[e] + t0.v[e]) : 0.f;
+    gz4[m] = addc(ldc<CW, true>(a.G + bL * 2 * S + CW * c), ldc<CW, false>(a.posG + CW * c));
+    gh4[m] = addc(ldc<CW, true>(a.G + bL * 2 * S + S + CW * c), ldc<CW, false>(a.posG + S + CW * c));
+    tz4[m] = ldc<CW, true>(a.Tzh + (size_t)x0 * 2 * S + CW * c);   // token share of x_{-1} = x0
+    th4[m] = ldc<CW, true>(a.Tzh + (size_t)x0 * 2 * S + S + CW * c);
   }
   float wgf[5];
 #pragma unroll
@@ -609,16 +647,16 @@ corrector_kernel(const __grid_constant__ ScanArgs a) {
   // them in the step.)
   constexpr bool PIPE = NP * CMC <= 16;
   constexpr int PK = PIPE ? NP : 1;
-  float4 ub[PK][CMC];
+  C ub[PK][CMC];
   if constexpr (PIPE) {
 #pragma unroll
     for (int k = 0; k < NP; ++k) {
       const float* Uk = a.U + (size_t)sm.cid[k < K ? k : K - 1] * S;
 #pragma unroll
-      for (int m = 0; m < CMC; ++m) ub[k][m] = ldcg4(Uk + 4 * cc[m]);
+      for (int m = 0; m < CMC; ++m) ub[k][m] = ldc<CW, true>(Uk + CW * cc[m]);
     }
   }
-  float4 tsz[CMC], tsh[CMC];                 // token share of the speculated previous token
+  C tsz[CMC], tsh[CMC];                      // token share of the speculated previous token
   int ts_id = -1;
 
   int prev = x0, prank = 0;
@@ -633,21 +671,21 @@ corrector_kernel(const __grid_constant__ ScanArgs a) {
       if (warp == NW - 1) prefetch_rows_l2(a.Tzh, ci + K, 0, 1, 1, 2 * S);
     }
     // into registers, for step i + 1: its residual rows and the rank-0 token-share row
-    float4 un[PK][CMC], tnz[CMC], tnh[CMC];
+    C un[PK][CMC], tnz[CMC], tnh[CMC];
     if (i + 1 < L) {
       if constexpr (PIPE) {
 #pragma unroll
         for (int k = 0; k < NP; ++k) {
           const float* Uk = a.U + (size_t)ci[K + (k < K ? k : K - 1)] * S;
 #pragma unroll
-          for (int m = 0; m < CMC; ++m) un[k][m] = ldcg4(Uk + 4 * cc[m]);
+          for (int m = 0; m < CMC; ++m) un[k][m] = ldc<CW, true>(Uk + CW * cc[m]);
         }
       }
       const float* Tn = a.Tzh + (size_t)ci[0] * 2 * S;
 #pragma unroll
       for (int m = 0; m < CMC; ++m) {
-        tnz[m] = ldcg4(Tn + 4 * cc[m]);
-        tnh[m] = ldcg4(Tn + S + 4 * cc[m]);
+        tnz[m] = ldc<CW, true>(Tn + CW * cc[m]);
+        tnh[m] = ldc<CW, true>(Tn + S + CW * cc[m]);
       }
     }
     // confidence features of position i (App. C.3)
@@ -671,8 +709,8 @@ corrector_kernel(const __grid_constant__ ScanArgs a) {
         const float* Tp = a.Tzh + (size_t)prev * 2 * S;
 #pragma unroll
         for (int m = 0; m < CMC; ++m) {
-          tz4[m] = ldcg4(Tp + 4 * cc[m]);
-          th4[m] = ldcg4(Tp + S + 4 * cc[m]);
+          tz4[m] = ldc<CW, true>(Tp + CW * cc[m]);
+          th4[m] = ldc<CW, true>(Tp + S + CW * cc[m]);
         }
       }
     }
@@ -681,35 +719,32 @@ corrector_kernel(const __grid_constant__ ScanArgs a) {
 #pragma unroll
     for (int m = 0; m < CMC; ++m) {
       const int c = cc[m];
-      float zp[4] = {gz4[m].x + tz4[m].x, gz4[m].y + tz4[m].y, gz4[m].z + tz4[m].z,
-                     gz4[m].w + tz4[m].w};
-      float hp[4] = {gh4[m].x + th4[m].x, gh4[m].y + th4[m].y, gh4[m].z + th4[m].z,
-                     gh4[m].w + th4[m].w};
-      // feature shares of this chunk's four elements: 20 contiguous floats of F[S, 5]
-      float fz[20], fh[20];
+      C zp = addc(gz4[m], tz4[m]), hp = addc(gh4[m], th4[m]);
+      // feature shares of this chunk's elements: 5 CW contiguous floats of F[S, 5]
+      float fz[5 * CW], fh[5 * CW];
 #pragma unroll
       for (int q = 0; q < 5; ++q) {
-        const float4 vz = ld4(sm.F + 20 * c + 4 * q);
-        const float4 vh = ld4(sm.F + 5 * S + 20 * c + 4 * q);
-        fz[4 * q] = vz.x; fz[4 * q + 1] = vz.y; fz[4 * q + 2] = vz.z; fz[4 * q + 3] = vz.w;
-        fh[4 * q] = vh.x; fh[4 * q + 1] = vh.y; fh[4 * q + 2] = vh.z; fh[4 * q + 3] = vh.w;
+        const C vz = ldc<CW, false>(sm.F + 5 * CW * c + CW * q);
+        const C vh = ldc<CW, false>(sm.F + 5 * S + 5 * CW * c + CW * q);
+#pragma unroll
+        for (int e = 0; e < CW; ++e) {
+          fz[CW * q + e] = vz.v[e];
+          fh[CW * q + e] = vh.v[e];
+        }
       }
 #pragma unroll
-      for (int e = 0; e < 4; ++e)
+      for (int e = 0; e < CW; ++e)
 #pragma unroll
         for (int f = 0; f < 5; ++f) {
-          zp[e] = fmaf(fz[5 * e + f], phi[f], zp[e]);
-          hp[e] = fmaf(fh[5 * e + f], phi[f], hp[e]);
+          zp.v[e] = fmaf(fz[5 * e + f], phi[f], zp.v[e]);
+          hp.v[e] = fmaf(fh[5 * e + f], phi[f], hp.v[e]);
         }
-      float sv[4] = {s4[m].x, s4[m].y, s4[m].z, s4[m].w};
 #pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const float z = sigmoid_fast(zp[e]);
-        sv[e] = ok[m] ? (1.f - z) * sv[e] + z * hp[e] : 0.f;
+      for (int e = 0; e < CW; ++e) {
+        const float z = sigmoid_fast(zp.v[e]);
+        s4[m].v[e] = ok[m] ? (1.f - z) * s4[m].v[e] + z * hp.v[e] : 0.f;
       }
-      s4[m] = make_float4(sv[0], sv[1], sv[2], sv[3]);
-      const float4 w4 = ld4(sm.wg + 4 * c);
-      gacc = fmaf(w4.x, sv[0], fmaf(w4.y, sv[1], fmaf(w4.z, sv[2], fmaf(w4.w, sv[3], gacc))));
+      gacc = dotc(ldc<CW, false>(sm.wg + CW * c), s4[m], gacc);
     }
     // residual-dot partials with the rows of this position's candidates
     float part[NP];
@@ -719,10 +754,10 @@ corrector_kernel(const __grid_constant__ ScanArgs a) {
       float acc = 0.f;
 #pragma unroll
       for (int m = 0; m < CMC; ++m) {
-        float4 u;
+        C u;
         if constexpr (PIPE) u = ub[k][m];
-        else u = ldcg4(Uk + 4 * cc[m]);
-        acc = fmaf(u.x, s4[m].x, fmaf(u.y, s4[m].y, fmaf(u.z, s4[m].z, fmaf(u.w, s4[m].w, acc))));
+        else u = ldc<CW, true>(Uk + CW * cc[m]);
+        acc = dotc(u, s4[m], acc);
       }
       part[k] = acc;
     }
@@ -732,8 +767,8 @@ corrector_kernel(const __grid_constant__ ScanArgs a) {
       const float* Pn = a.posG + (size_t)(i + 1) * 2 * S;
 #pragma unroll
       for (int m = 0; m < CMC; ++m) {
-        gz4[m] = add4(ldcg4(Gn + 4 * cc[m]), ld4(Pn + 4 * cc[m]));
-        gh4[m] = add4(ldcg4(Gn + S + 4 * cc[m]), ld4(Pn + S + 4 * cc[m]));
+        gz4[m] = addc(ldc<CW, true>(Gn + CW * cc[m]), ldc<CW, false>(Pn + CW * cc[m]));
+        gh4[m] = addc(ldc<CW, true>(Gn + S + CW * cc[m]), ldc<CW, false>(Pn + S + CW * cc[m]));
       }
     }
     // residual dots by a warp reduce-scatter; across warps through shared memory
@@ -815,40 +850,41 @@ size_t scan_smem_bytes(int L, int K, int S, int V) {
   return smem_layout(L, K, S, V, nullptr, nullptr);
 }
 
-template <int NW, int NP, int CMC, bool VERIFY>
+template <int NW, int NP, int CMC, int CW, bool VERIFY>
 cudaError_t launch_corrector_k(const ScanArgs& a, cudaStream_t stream) {
   const size_t smem = corr_layout(a.L, a.K, a.S, NW, a.V, VERIFY, nullptr, nullptr);
-  cudaError_t e = cudaFuncSetAttribute(corrector_kernel<NW, NP, CMC, VERIFY>,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  if (e == cudaSuccess) e = prefer_carveout(corrector_kernel<NW, NP, CMC, VERIFY>, CARVEOUT_SMALL_KB);
+  auto kernel = corrector_kernel<NW, NP, CMC, CW, VERIFY>;
+  cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e == cudaSuccess) e = prefer_carveout(kernel, CARVEOUT_SMALL_KB);
   if (e != cudaSuccess) return e;
-  e = launch_prio(corrector_kernel<NW, NP, CMC, VERIFY>, dim3(a.B), dim3(NW * 32), smem, stream, a);
+  e = launch_prio(kernel, dim3(a.B), dim3(NW * 32), smem, stream, a);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 
-template <int NP, int CMC, int NW = CORR_WARPS>
+template <int NW, int CW, int NP>
 cudaError_t launch_corrector(const ScanArgs& a, cudaStream_t stream) {
-  if (a.do_verify) return launch_corrector_k<NW, NP, CMC, true>(a, stream);
-  return launch_corrector_k<NW, NP, CMC, false>(a, stream);
+  if (a.do_verify) return launch_corrector_k<NW, NP, 1, CW, true>(a, stream);
+  return launch_corrector_k<NW, NP, 1, CW, false>(a, stream);
+}
+
+template <int NW, int CW>
+cudaError_t launch_corrector_for_k(const ScanArgs& a, cudaStream_t stream) {
+  if (a.K <= 8) return launch_corrector<NW, CW, 8>(a, stream);
+  return a.K <= 16 ? launch_corrector<NW, CW, 16>(a, stream) : launch_corrector<NW, CW, 32>(a, stream);
 }
 
 // The corrector (do_select; with do_verify also the verification in the same CTA) or the
 // verification alone (do_verify) for every sequence.
 cudaError_t launch_scan(const ScanArgs& a, cudaStream_t stream) {
   if (a.do_select) {
-    // 4-element chunks per lane: S / 4 chunks over the CTA's lanes. A state wider than four
-    // warps' chunks (S > 512, up to 1024) takes eight warps, one chunk a lane, rather than two
-    // chunks a lane: the next position's residual rows then fit the register pipeline, and each
-    // SM sub-partition has two warps of the sequence to issue from (large_vocab, S = 1024,
-    // K = 16: products and corrector 535 -> 284 us, step 856 -> 604 us).
-    if (a.S > 4 * 32 * CORR_WARPS) {
-      if (a.K <= 8) return launch_corrector<8, 1, 2 * CORR_WARPS>(a, stream);
-      return a.K <= 16 ? launch_corrector<16, 1, 2 * CORR_WARPS>(a, stream)
-                       : launch_corrector<32, 1, 2 * CORR_WARPS>(a, stream);
-    }
-    if (a.K <= 8) return launch_corrector<8, 1>(a, stream);
-    return a.K <= 16 ? launch_corrector<16, 1>(a, stream) : launch_corrector<32, 1>(a, stream);
+    // One chunk a lane. Up to S = 512 four warps of 4-element chunks, one warp per SM
+    // sub-partition; a state of 257..512 takes eight warps of 2-element chunks instead, and a
+    // wider one (up to 1024) eight warps of 4-element chunks: two warps of the sequence on each
+    // sub-partition to issue from, and half a position's dependent element work a lane.
+    if (a.S > 4 * 32 * CORR_WARPS) return launch_corrector_for_k<2 * CORR_WARPS, 4>(a, stream);
+    if (a.S > 4 * 32 * CORR_WARPS / 2) return launch_corrector_for_k<2 * CORR_WARPS, 2>(a, stream);
+    return launch_corrector_for_k<CORR_WARPS, 4>(a, stream);
   }
   const size_t smem = scan_smem_bytes(a.L, a.K, a.S, a.V);
   cudaError_t e = cudaFuncSetAttribute(verify_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
