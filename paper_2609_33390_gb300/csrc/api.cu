@@ -656,8 +656,9 @@ brisk_status brisk::decode_tail_locked(const brisk_dims* d, const brisk_params* 
   // verifier rows on the low-priority stream
   if (ev && ev->sweep_p_begin) BRISK_CUDA(cudaEventRecord(static_cast<cudaEvent_t>(ev->sweep_p_begin), ss->lo));
   BRISK_CUDA(launch_sweep(sp, ss->lo));
-  if (ev && ev->sweep_p_end) BRISK_CUDA(cudaEventRecord(static_cast<cudaEvent_t>(ev->sweep_p_end), ss->lo));
+  // the join first: a timing record ahead of it would delay the verification behind it
   BRISK_CUDA(cudaEventRecord(ss->ev[3], ss->lo));
+  if (ev && ev->sweep_p_end) BRISK_CUDA(cudaEventRecord(static_cast<cudaEvent_t>(ev->sweep_p_end), ss->lo));
 
   // the corrector once the proposal candidates and the hidden products are done
   BRISK_CUDA(cudaStreamWaitEvent(m, ss->ev[1], 0));

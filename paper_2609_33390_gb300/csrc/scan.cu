@@ -75,7 +75,7 @@ __device__ __forceinline__ float4 ldcg4(const float* p) {
   return __ldcg(reinterpret_cast<const float4*>(p));
 }
 
-// A lane's chunk of CW consecutive state elements (CW = 2 or 4), loaded as one vector.
+// A lane's chunk of CW consecutive state elements (CW = 1, 2 or 4), loaded as one vector.
 template <int CW>
 struct Chunk {
   float v[CW];
@@ -90,10 +90,12 @@ __device__ __forceinline__ Chunk<CW> ldc(const float* p) {
   if constexpr (CW == 4) {
     return chunk_of<4>(CG ? __ldcg(reinterpret_cast<const float4*>(p))
                           : *reinterpret_cast<const float4*>(p));
-  } else {
+  } else if constexpr (CW == 2) {
     const float2 t = CG ? __ldcg(reinterpret_cast<const float2*>(p))
                         : *reinterpret_cast<const float2*>(p);
     return {{t.x, t.y}};
+  } else {
+    return {{CG ? __ldcg(p) : *p}};
   }
 }
 template <int CW>
@@ -546,7 +548,7 @@ __device__ __forceinline__ void gather_logits(const void* logits, int dt, int n,
 }
 
 // The sequential corrector (Sec. 3.3 Eqs. 4-5; App. C.3 Eq. 9; Algorithm 1(b) loop), one CTA of
-// NW warps per sequence. Lane l of warp w owns the CW-element state chunks (CW = 2 or 4)
+// NW warps per sequence. Lane l of warp w owns the CW-element state chunks (CW = 1, 2 or 4)
 // c = l + 32 (w + NW m), m < CMC. The residual dots and the gate are reduced with warp
 // shuffles, then across the warps through shared memory (one block barrier a position), and
 // Select runs in every warp with lane k holding candidate k. Spreading a sequence over the
@@ -641,8 +643,10 @@ corrector_kernel(const __grid_constant__ ScanArgs a) {
   __syncthreads();
 
   // Software pipeline across positions: the next position's residual rows (rank K-1 repeated
-  // past K) are loaded into registers one step ahead, and so is the token-share row of this
-  // position's rank-0 candidate, the usual next previous token.
+  // past K) and hidden and position shares are loaded into registers one step ahead (issued at
+  // the top of the step: issued after the step's dots they were still in flight when the next
+  // step began, single 118 -> 110 us for the products and the corrector), and so is the
+  // token-share row of this position's rank-0 candidate, the usual next previous token.
   // (Only while the rows fit in registers: NP * CMC <= 16 vectors a lane; wider variants load
   // them in the step.)
   constexpr bool PIPE = NP * CMC <= 16;
@@ -670,9 +674,19 @@ corrector_kernel(const __grid_constant__ ScanArgs a) {
       prefetch_rows_l2(a.U, ci + 2 * K, warp, NW, K, S);
       if (warp == NW - 1) prefetch_rows_l2(a.Tzh, ci + K, 0, 1, 1, 2 * S);
     }
-    // into registers, for step i + 1: its residual rows and the rank-0 token-share row
-    C un[PK][CMC], tnz[CMC], tnh[CMC];
+    // into registers, for step i + 1: its hidden and position shares, residual rows and the
+    // rank-0 token-share row
+    C un[PK][CMC], tnz[CMC], tnh[CMC], gnz[CMC], gnh[CMC], pnz[CMC], pnh[CMC];
     if (i + 1 < L) {
+      const float* Gn = a.G + (bL + i + 1) * 2 * S;
+      const float* Pn = a.posG + (size_t)(i + 1) * 2 * S;
+#pragma unroll
+      for (int m = 0; m < CMC; ++m) {
+        gnz[m] = ldc<CW, true>(Gn + CW * cc[m]);
+        gnh[m] = ldc<CW, true>(Gn + S + CW * cc[m]);
+        pnz[m] = ldc<CW, false>(Pn + CW * cc[m]);
+        pnh[m] = ldc<CW, false>(Pn + S + CW * cc[m]);
+      }
       if constexpr (PIPE) {
 #pragma unroll
         for (int k = 0; k < NP; ++k) {
@@ -763,12 +777,10 @@ corrector_kernel(const __grid_constant__ ScanArgs a) {
     }
     // hidden and position shares of the next position: plain loads first used in the next step
     if (i + 1 < L) {
-      const float* Gn = a.G + (bL + i + 1) * 2 * S;
-      const float* Pn = a.posG + (size_t)(i + 1) * 2 * S;
 #pragma unroll
       for (int m = 0; m < CMC; ++m) {
-        gz4[m] = addc(ldc<CW, true>(Gn + CW * cc[m]), ldc<CW, false>(Pn + CW * cc[m]));
-        gh4[m] = addc(ldc<CW, true>(Gn + S + CW * cc[m]), ldc<CW, false>(Pn + S + CW * cc[m]));
+        gz4[m] = addc(gnz[m], pnz[m]);
+        gh4[m] = addc(gnh[m], pnh[m]);
       }
     }
     // residual dots by a warp reduce-scatter; across warps through shared memory
@@ -878,13 +890,16 @@ cudaError_t launch_corrector_for_k(const ScanArgs& a, cudaStream_t stream) {
 // verification alone (do_verify) for every sequence.
 cudaError_t launch_scan(const ScanArgs& a, cudaStream_t stream) {
   if (a.do_select) {
-    // One chunk a lane. Up to S = 512 four warps of 4-element chunks, one warp per SM
-    // sub-partition; a state of 257..512 takes eight warps of 2-element chunks instead, and a
+    // One chunk a lane. A state of up to 256 takes four warps, one per SM sub-partition, of
+    // 1- or 2-element chunks (every lane busy); 257..512 eight warps of 2-element chunks and a
     // wider one (up to 1024) eight warps of 4-element chunks: two warps of the sequence on each
-    // sub-partition to issue from, and half a position's dependent element work a lane.
+    // sub-partition to issue from. (At S = 512 eight warps of 2-element chunks beat four of
+    // 4-element chunks, single 144 -> 135 us a tail, and sixteen of single elements, 138 us:
+    // the cross-warp sums grow with the warps.)
     if (a.S > 4 * 32 * CORR_WARPS) return launch_corrector_for_k<2 * CORR_WARPS, 4>(a, stream);
-    if (a.S > 4 * 32 * CORR_WARPS / 2) return launch_corrector_for_k<2 * CORR_WARPS, 2>(a, stream);
-    return launch_corrector_for_k<CORR_WARPS, 4>(a, stream);
+    if (a.S > 2 * 32 * CORR_WARPS) return launch_corrector_for_k<2 * CORR_WARPS, 2>(a, stream);
+    if (a.S > 32 * CORR_WARPS) return launch_corrector_for_k<CORR_WARPS, 2>(a, stream);
+    return launch_corrector_for_k<CORR_WARPS, 1>(a, stream);
   }
   const size_t smem = scan_smem_bytes(a.L, a.K, a.S, a.V);
   cudaError_t e = cudaFuncSetAttribute(verify_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,

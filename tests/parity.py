@@ -91,8 +91,10 @@ def check_sequence(b: int, block: dict, params: O.Params, K: int, gpu: dict, sel
             u_sel, u_acc, u_res, force_sel, force_acc, force_corr)
         # step 1: candidates (no near-ties possible: exact comparisons of exact values)
         np.testing.assert_array_equal(gpu["cand_ids"][b], cand, err_msg=f"cand_ids seq {b}")
-        e = np.abs(gpu["cand_logprob"][b] - lp)
-        e = np.where(np.isfinite(lp), e, 0.0)
+        fin = np.isfinite(lp)   # a candidate of zero mass (K > support) is -inf on both sides
+        np.testing.assert_array_equal(gpu["cand_logprob"][b][~fin], lp[~fin],
+                                      err_msg=f"cand_logprob seq {b}")
+        e = np.where(fin, np.abs(gpu["cand_logprob"][b] - np.where(fin, lp, 0.0)), 0.0)
         rep.max_lp_err = max(rep.max_lp_err, float(e.max()))
         assert e.max() <= ATOL, f"cand_logprob seq {b}: {e.max()}"
         el = float(np.abs(gpu["lse_q"][b] - lse).max())

@@ -79,6 +79,13 @@ SMALL = [
                                   verify_mode="stochastic", weight_std=0.06)),
     ("wide_state_k16", dict(B=2, L=7, V=2500, d=64, K=16, r=384, weight_std=0.06)),
     ("wide_state_k32", dict(B=2, L=6, V=3000, d=64, K=32, r=512, weight_std=0.06)),
+    # 2-element chunks: four warps (S = 192, chunks ending inside the third warp; S = 256) and
+    # eight warps (S = 512) in the K classes the workloads do not reach
+    ("state192_k16", dict(B=2, L=6, V=2200, d=64, K=16, r=96, weight_std=0.1)),
+    ("state256_k32_sample", dict(B=2, L=5, V=2600, d=64, K=32, r=128, select_mode="sample",
+                                 verify_mode="stochastic", weight_std=0.1)),
+    ("state512_k16", dict(B=2, L=6, V=2400, d=64, K=16, r=256, weight_std=0.06)),
+    ("state512_k32", dict(B=2, L=5, V=3100, d=64, K=32, r=256, weight_std=0.06)),
 ]
 
 
