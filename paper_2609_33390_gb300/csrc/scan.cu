@@ -66,16 +66,10 @@ __host__ __device__ inline size_t smem_layout(int L, int K, int S, int V, char* 
 }
 
 __device__ __forceinline__ float4 ld4(const float* p) { return *reinterpret_cast<const float4*>(p); }
-__device__ __forceinline__ float4 add4(float4 x, float4 y) {
-  return make_float4(x.x + y.x, x.y + y.y, x.z + y.z, x.w + y.w);
-}
-// Cached in L2 only: rows read once per step must not displace the L1 lines that hold a
-// concurrent streaming kernel's loads in flight.
-__device__ __forceinline__ float4 ldcg4(const float* p) {
-  return __ldcg(reinterpret_cast<const float4*>(p));
-}
 
-// A lane's chunk of CW consecutive state elements (CW = 1, 2 or 4), loaded as one vector.
+// A lane's chunk of CW consecutive state elements (CW = 1, 2 or 4), loaded as one vector;
+// CG: cached in L2 only (rows read once per step must not displace the L1 lines that hold a
+// concurrent streaming kernel's loads in flight).
 template <int CW>
 struct Chunk {
   float v[CW];
@@ -556,12 +550,14 @@ __device__ __forceinline__ void gather_logits(const void* logits, int dt, int n,
 // sub-partition's share small, so the verifier-row sweep beside it keeps its issue slots.
 // Every load of the step is issued unconditionally (chunk and candidate indices clamped into
 // range, the surplus contributions multiplied by zero state or never read) so the compiler can
-// keep them all in flight. Candidate rows are read through L2, prefetched two positions ahead;
-// shared memory holds only small per-sequence tables.
+// keep them all in flight. Table rows are read through L2 (cache-global loads) a whole position
+// ahead into registers; an L2 line prefetch two positions ahead on top of that was slower
+// (single 105.7 -> 102.5 us for the products and the corrector without it, large_vocab
+// 269 -> 253 us). Shared memory holds only small per-sequence tables.
 // VERIFY: the CTA also verifies its sequence after the scan (the fused small-batch schedule); a
-// separate instantiation, since the verification code raises the scan's register count (168 ->
-// 228 a thread for four warps and K = 8), which would leave less room for the verifier-row
-// sweep beside the corrector in the overlapping schedule.
+// separate instantiation, since the verification code raises the scan's register count (123 ->
+// 164 a thread for four warps of 2-element chunks and K = 8), which would leave less room for
+// the verifier-row sweep beside the corrector in the overlapping schedule.
 template <int NW, int NP, int CMC, int CW, bool VERIFY>
 __global__ void __launch_bounds__(NW * 32)
 corrector_kernel(const __grid_constant__ ScanArgs a) {
@@ -639,6 +635,29 @@ corrector_kernel(const __grid_constant__ ScanArgs a) {
   float wgf[5];
 #pragma unroll
   for (int f = 0; f < 5; ++f) wgf[f] = a.wg[S + f];
+  // chunks of up to two elements: this lane's feature shares (5 CW floats of F[S, 5] for z and
+  // for h) and gate weights, read every step, held in registers for the whole scan (4-element
+  // chunks read them from shared memory: in registers they would spill)
+  constexpr bool FREG = CW <= 2;
+  constexpr int FR = FREG ? CMC : 1;
+  float fzr[FR][5 * CW], fhr[FR][5 * CW];
+  C wgr[FR];
+  if constexpr (FREG) {
+#pragma unroll
+    for (int m = 0; m < CMC; ++m) {
+#pragma unroll
+      for (int q = 0; q < 5; ++q) {
+        const C vz = ldc<CW, false>(a.Fz + 5 * CW * cc[m] + CW * q);
+        const C vh = ldc<CW, false>(a.Fh + 5 * CW * cc[m] + CW * q);
+#pragma unroll
+        for (int e = 0; e < CW; ++e) {
+          fzr[m][CW * q + e] = vz.v[e];
+          fhr[m][CW * q + e] = vh.v[e];
+        }
+      }
+      wgr[m] = ldc<CW, false>(a.wg + CW * cc[m]);
+    }
+  }
   const float sig_alpha = sigmoidf_(a.alpha);
   __syncthreads();
 
@@ -668,12 +687,6 @@ corrector_kernel(const __grid_constant__ ScanArgs a) {
   for (int i = 0; i < L; ++i) {
     const int buf = i & 1;
     const int* ci = sm.cid + i * K;
-    // into L2, for step i + 2: its residual rows, and the token-share row of the next
-    // position's rank-0 candidate
-    if (i + 2 < L) {
-      prefetch_rows_l2(a.U, ci + 2 * K, warp, NW, K, S);
-      if (warp == NW - 1) prefetch_rows_l2(a.Tzh, ci + K, 0, 1, 1, 2 * S);
-    }
     // into registers, for step i + 1: its hidden and position shares, residual rows and the
     // rank-0 token-share row
     C un[PK][CMC], tnz[CMC], tnh[CMC], gnz[CMC], gnh[CMC], pnz[CMC], pnh[CMC];
@@ -736,14 +749,22 @@ corrector_kernel(const __grid_constant__ ScanArgs a) {
       C zp = addc(gz4[m], tz4[m]), hp = addc(gh4[m], th4[m]);
       // feature shares of this chunk's elements: 5 CW contiguous floats of F[S, 5]
       float fz[5 * CW], fh[5 * CW];
+      if constexpr (FREG) {
 #pragma unroll
-      for (int q = 0; q < 5; ++q) {
-        const C vz = ldc<CW, false>(sm.F + 5 * CW * c + CW * q);
-        const C vh = ldc<CW, false>(sm.F + 5 * S + 5 * CW * c + CW * q);
+        for (int j = 0; j < 5 * CW; ++j) {
+          fz[j] = fzr[m][j];
+          fh[j] = fhr[m][j];
+        }
+      } else {
 #pragma unroll
-        for (int e = 0; e < CW; ++e) {
-          fz[CW * q + e] = vz.v[e];
-          fh[CW * q + e] = vh.v[e];
+        for (int q = 0; q < 5; ++q) {
+          const C vz = ldc<CW, false>(sm.F + 5 * CW * c + CW * q);
+          const C vh = ldc<CW, false>(sm.F + 5 * S + 5 * CW * c + CW * q);
+#pragma unroll
+          for (int e = 0; e < CW; ++e) {
+            fz[CW * q + e] = vz.v[e];
+            fh[CW * q + e] = vh.v[e];
+          }
         }
       }
 #pragma unroll
@@ -758,7 +779,8 @@ corrector_kernel(const __grid_constant__ ScanArgs a) {
         const float z = sigmoid_fast(zp.v[e]);
         s4[m].v[e] = ok[m] ? (1.f - z) * s4[m].v[e] + z * hp.v[e] : 0.f;
       }
-      gacc = dotc(ldc<CW, false>(sm.wg + CW * c), s4[m], gacc);
+      if constexpr (FREG) gacc = dotc(wgr[m], s4[m], gacc);
+      else gacc = dotc(ldc<CW, false>(sm.wg + CW * c), s4[m], gacc);
     }
     // residual-dot partials with the rows of this position's candidates
     float part[NP];
