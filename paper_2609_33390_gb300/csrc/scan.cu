@@ -493,19 +493,6 @@ __host__ __device__ inline size_t corr_layout(int L, int K, int S, int NW, int V
   return off;
 }
 
-// Brings rows k = k0, k0 + kstep, ... < K of `row_floats` floats at table + ids[k] * row_floats
-// into L2 without waiting: one 128-byte line per lane and instruction. (Line prefetches disturb
-// a concurrent streaming kernel far less than bulk prefetches of whole rows.)
-__device__ __forceinline__ void prefetch_rows_l2(const float* table, const int* ids, int k0, int kstep,
-                                                 int K, int row_floats) {
-  const int lane = threadIdx.x & 31;
-  const int lines = row_floats / 32;
-  for (int k = k0; k < K; k += kstep) {
-    const float* row = table + (size_t)ids[k] * row_floats;
-    for (int l = lane; l < lines; l += 32) asm volatile("prefetch.global.L2 [%0];" ::"l"(row + 32 * l));
-  }
-}
-
 // Warp reduce-scatter of NP values per lane (NP = 8, 16 or 32): afterwards lane l holds the
 // warp-wide sum of value (l >> log2(32 / NP)) & (NP - 1), that is value k sits in lane
 // k * (32 / NP).
@@ -528,10 +515,10 @@ __device__ __forceinline__ float reduce_scatter_n(float (&v)[NP]) {
   return r;
 }
 
-// Gathers logits at nidx (row, column) pairs into dst, eight loads in flight per lane.
-template <int NT, typename IndexOf>
-__device__ __forceinline__ void gather_logits(const void* logits, int dt, int n, float* dst,
-                                              IndexOf index_of) {
+// Gathers n logits, entry e at index_of(e) into *dst_of(e), eight loads in flight per lane.
+template <int NT, typename IndexOf, typename DstOf>
+__device__ __forceinline__ void gather_logits(const void* logits, int dt, int n, IndexOf index_of,
+                                              DstOf dst_of) {
   const int tid = threadIdx.x;
   for (int base = 0; base < n; base += 8 * NT) {
     float v[8];
@@ -543,7 +530,7 @@ __device__ __forceinline__ void gather_logits(const void* logits, int dt, int n,
 #pragma unroll
     for (int j = 0; j < 8; ++j) {
       const int e = base + j * NT + tid;
-      if (e < n) dst[e] = v[j];
+      if (e < n) *dst_of(e) = v[j];
     }
   }
 }
@@ -579,42 +566,10 @@ corrector_kernel(const __grid_constant__ ScanArgs a) {
   const size_t bL = (size_t)b * L;
   const int nch = S / CW;
 
-  for (int e = tid; e < L * K; e += NT) {
-    int c = a.cand_ids[bL * K + e];
-    if (c < 0 || c >= V) { set_status(a.status, BRISK_ERR_NUMERIC); c = 0; }
-    sm.cid[e] = c;
-    sm.clp[e] = a.cand_logprob[bL * K + e];
-  }
-  int x0 = a.x0[b];
-  if (x0 < 0 || x0 >= V) {
-    if (tid == 0) set_status(a.status, BRISK_ERR_INVALID_ARG);
-    x0 = 0;
-  }
-  // the feature shares and the gate weights, read every step, into shared memory
-  for (int e = tid; e < 5 * S / 4; e += NT) {
-    reinterpret_cast<float4*>(sm.F)[e] = ld4(a.Fz + 4 * e);
-    reinterpret_cast<float4*>(sm.F + 5 * S)[e] = ld4(a.Fh + 4 * e);
-  }
-  for (int e = tid; e < S / 4; e += NT) reinterpret_cast<float4*>(sm.wg)[e] = ld4(a.wg + 4 * e);
-  __syncthreads();
-  // into L2: the first two positions' residual rows, and the token-share row of the first
-  // position's rank-0 candidate (the usual next previous token; others are fetched on demand,
-  // since speculative rows for every rank would cost the concurrent sweep far more DRAM
-  // bandwidth than the rare miss costs here)
-  prefetch_rows_l2(a.U, sm.cid, warp, NW, K * (L > 1 ? 2 : 1), S);
-  if (L > 1 && warp == NW - 1) prefetch_rows_l2(a.Tzh, sm.cid, 0, 1, 1, 2 * S);
-  // the features' logit gathers, all independent of the selections
-  const void* lq = a.logits_q;
-  const int ldt = a.logits_dt;
-  gather_logits<NT>(lq, ldt, L * 3, sm.top, [&](int e) {
-    const int i = e / 3, w = e % 3;
-    return (bL + i) * V + sm.cid[i * K + (w == 0 ? 0 : (w == 1 ? 1 : 3))];
-  });
-  gather_logits<NT>(lq, ldt, L * K, sm.lprev, [&](int e) {
-    const int i = e / K, k = e % K;
-    return i == 0 ? bL * V + x0 : (bL + i) * V + sm.cid[(i - 1) * K + k];
-  });
-
+  // Prologue in two dependent rounds of loads. First everything that depends neither on the
+  // candidates nor on x0, issued at once with the candidate table itself; then, after one
+  // barrier, what depends on them (the token shares of x0, the first position's residual rows
+  // and the features' logit gathers, in one batch).
   // lane chunks, clamped into range; a chunk past the state keeps s = 0 throughout
   int cc[CMC];
   bool ok[CMC];
@@ -625,19 +580,17 @@ corrector_kernel(const __grid_constant__ ScanArgs a) {
     cc[m] = ok[m] ? c : nch - 1;
   }
   using C = Chunk<CW>;
-  C s4[CMC], gz4[CMC], gh4[CMC], tz4[CMC], th4[CMC];
+  int x0 = a.x0[b];
+  // the Init share of h_c and the first position's hidden and position shares
+  C g0c[CMC], gz4[CMC], gh4[CMC], pz0[CMC], ph0[CMC];
 #pragma unroll
   for (int m = 0; m < CMC; ++m) {
     const int c = cc[m];
-    const C g0 = ldc<CW, true>(a.G0 + (size_t)b * S + CW * c);
-    const C t0 = ldc<CW, true>(a.T0 + (size_t)x0 * S + CW * c);
-#pragma unroll
-    for (int e = 0; e < CW; ++e)                              // s_{-1} = u_0 = Init(h_c, E(x0))
-      s4[m].v[e] = ok[m] ? tanhf(g0.v[e] + t0.v[e]) : 0.f;
-    gz4[m] = addc(ldc<CW, true>(a.G + bL * 2 * S + CW * c), ldc<CW, false>(a.posG + CW * c));
-    gh4[m] = addc(ldc<CW, true>(a.G + bL * 2 * S + S + CW * c), ldc<CW, false>(a.posG + S + CW * c));
-    tz4[m] = ldc<CW, true>(a.Tzh + (size_t)x0 * 2 * S + CW * c);   // token share of x_{-1} = x0
-    th4[m] = ldc<CW, true>(a.Tzh + (size_t)x0 * 2 * S + S + CW * c);
+    g0c[m] = ldc<CW, true>(a.G0 + (size_t)b * S + CW * c);
+    gz4[m] = ldc<CW, true>(a.G + bL * 2 * S + CW * c);
+    gh4[m] = ldc<CW, true>(a.G + bL * 2 * S + S + CW * c);
+    pz0[m] = ldc<CW, false>(a.posG + CW * c);
+    ph0[m] = ldc<CW, false>(a.posG + S + CW * c);
   }
   float wgf[5];
 #pragma unroll
@@ -666,6 +619,71 @@ corrector_kernel(const __grid_constant__ ScanArgs a) {
     }
   }
   const float sig_alpha = sigmoidf_(a.alpha);
+  // the candidate table
+  for (int e = tid; e < L * K; e += NT) {
+    int c = a.cand_ids[bL * K + e];
+    if (c < 0 || c >= V) { set_status(a.status, BRISK_ERR_NUMERIC); c = 0; }
+    sm.cid[e] = c;
+    sm.clp[e] = a.cand_logprob[bL * K + e];
+  }
+  if (x0 < 0 || x0 >= V) {
+    if (tid == 0) set_status(a.status, BRISK_ERR_INVALID_ARG);
+    x0 = 0;
+  }
+  if constexpr (!FREG) {
+    // the feature shares and the gate weights into shared memory, all loads first
+    constexpr int FV = 2 * 5 * 1024 / 4 / NT + 1;   // float4 of Fz and Fh a thread, S <= 1024
+    float4 fv[FV];
+    const int nf = 5 * S / 4;
+#pragma unroll
+    for (int j = 0; j < FV; ++j) {
+      const int e = tid + j * NT;
+      fv[j] = e < nf ? ld4(a.Fz + 4 * e) : (e < 2 * nf ? ld4(a.Fh + 4 * (e - nf)) : float4{});
+    }
+    const float4 wv = tid < S / 4 ? ld4(a.wg + 4 * tid) : float4{};
+#pragma unroll
+    for (int j = 0; j < FV; ++j) {
+      const int e = tid + j * NT;
+      if (e < 2 * nf) reinterpret_cast<float4*>(sm.F)[e] = fv[j];
+    }
+    for (int e = tid; e < S / 4; e += NT)
+      reinterpret_cast<float4*>(sm.wg)[e] = e == tid ? wv : ld4(a.wg + 4 * e);
+  }
+  __syncthreads();
+
+  // second round: the token shares of x0, the first position's residual rows (below) and the
+  // features' logit gathers, all independent of the selections
+  C t0c[CMC], tz4[CMC], th4[CMC];
+#pragma unroll
+  for (int m = 0; m < CMC; ++m) {
+    const int c = cc[m];
+    t0c[m] = ldc<CW, true>(a.T0 + (size_t)x0 * S + CW * c);
+    tz4[m] = ldc<CW, true>(a.Tzh + (size_t)x0 * 2 * S + CW * c);   // token share of x_{-1} = x0
+    th4[m] = ldc<CW, true>(a.Tzh + (size_t)x0 * 2 * S + S + CW * c);
+  }
+  const void* lq = a.logits_q;
+  const int ldt = a.logits_dt;
+  gather_logits<NT>(
+      lq, ldt, L * 3 + L * K,
+      [&](int e) {
+        if (e < L * 3) {
+          const int i = e / 3, w = e % 3;
+          return (bL + i) * V + sm.cid[i * K + (w == 0 ? 0 : (w == 1 ? 1 : 3))];
+        }
+        e -= L * 3;
+        const int i = e / K, k = e % K;
+        return i == 0 ? bL * V + x0 : (bL + i) * V + sm.cid[(i - 1) * K + k];
+      },
+      [&](int e) { return e < L * 3 ? sm.top + e : sm.lprev + (e - L * 3); });
+  C s4[CMC];
+#pragma unroll
+  for (int m = 0; m < CMC; ++m) {
+#pragma unroll
+    for (int e = 0; e < CW; ++e)                              // s_{-1} = u_0 = Init(h_c, E(x0))
+      s4[m].v[e] = ok[m] ? tanhf(g0c[m].v[e] + t0c[m].v[e]) : 0.f;
+    gz4[m] = addc(gz4[m], pz0[m]);
+    gh4[m] = addc(gh4[m], ph0[m]);
+  }
   __syncthreads();
 
   // Software pipeline across positions: the next position's residual rows (rank K-1 repeated
