@@ -213,7 +213,13 @@ brisk_status brisk_verify_block(const brisk_dims *dims, const void *logits_p,
  * join back to it, also under graph capture). The first call in a CUDA context creates the side
  * streams and their events: make it before any stream capture. Calls from several host threads
  * are serialised while they enqueue, and brisk_tail_graph_create holds that serialisation for
- * the whole of its capture. `ev` may be NULL. */
+ * the whole of its capture. `ev` may be NULL.
+ * logits_q and logits_p may also point to page-locked host memory (cudaHostAlloc /
+ * cudaMallocHost, or cudaHostRegister with cudaHostRegisterMapped; mapped into the device's
+ * unified address space): the kernels then read the logits in place over the host link, with
+ * the same results bit for bit (about 210 GB/s on a GB300 with its Grace host, the rate of a
+ * copy-engine copy of the same buffers, without the copy's second pass through HBM). Every
+ * other pointer is device memory; memory that is neither is undefined behaviour. */
 brisk_status brisk_decode_tail(const brisk_dims *dims, const brisk_params *params,
                                const void *tables, const brisk_tail_io *io, int32_t select_mode,
                                int32_t verify_mode, void *workspace, const brisk_events *ev,
