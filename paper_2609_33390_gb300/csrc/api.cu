@@ -184,8 +184,12 @@ SweepSeg make_seg(const WsLayout& w, void* ws, int seg, const void* logits, int 
 // column tiles and a 4-deep pipeline (four times the CTAs, each streaming a quarter of the
 // weights). With `wide` (large batches, the products running beside the proposal sweep) it uses
 // 256-wide tiles and a 2-deep pipeline: a quarter of the CTAs, so the sweep waits for fewer SMs,
-// and the hidden states are read once. Tile width does not change any product's summation
-// order, so both give the same bits.
+// and the hidden states are read once; or, where the second product is small (S <= 512), both
+// products in 64-wide tiles and a 2-deep pipeline that fit the sweep's shared-memory carveout,
+// so that their CTAs share SMs with sweep CTAs instead of holding SMs of their own (decode_stream
+// 395 -> 392 us a step; large_vocab's four times larger second product: 561 -> 601 us, not
+// used there). Tile width does not change any product's summation order, so all give the same
+// bits.
 brisk_status hidden_products(const brisk_dims* d, const brisk_params* p, const void* tables,
                              const void* hidden, const void* h_ctx, const WsLayout& w, void* ws,
                              cudaStream_t st, bool wide) {
@@ -196,17 +200,18 @@ brisk_status hidden_products(const brisk_dims* d, const brisk_params* p, const v
       aligned(h_ctx, 16)) {
     __nv_bfloat16* Hs = at<__nv_bfloat16>(ws, w.Hm);   // [BL + B, 3r]: hi | mid | lo
     const int r3 = 3 * r;
-    const int bn = wide ? 256 : 64;
+    const bool share = wide && S <= 512;   // tiles that fit the sweep's carveout
+    const int bn = wide && !share ? 256 : 64;
     const TcSpec first[2] = {
         {BL, r, d->d, hidden, d->d, p->P_h, d->d, 1, Hs, r3, nullptr, 0, bn},
         {d->B, r, d->d, h_ctx, d->d, p->P_h, d->d, 1, Hs + (size_t)BL * r3, r3, nullptr, 0, bn}};
-    BRISK_CUDA(gemm_tc_grouped(first, 2, status, st, wide ? 2 : 4));
+    BRISK_CUDA(gemm_tc_grouped(first, 2, status, st, wide ? 2 : 4, share));
     const TcSpec second[2] = {
         {BL, 2 * S, r3, Hs, r3, at<__nv_bfloat16>(tables, t.W2s), r3, 0, at<float>(ws, w.G), 2 * S,
-         nullptr, 0, 0},
+         nullptr, 0, share ? 64 : 0},
         {d->B, S, r3, Hs + (size_t)BL * r3, r3, at<__nv_bfloat16>(tables, t.W0s), r3, 0,
-         at<float>(ws, w.G0), S, nullptr, 0, 0}};
-    BRISK_CUDA(gemm_tc_grouped(second, 2, status, st, 2));
+         at<float>(ws, w.G0), S, nullptr, 0, share ? 64 : 0}};
+    BRISK_CUDA(gemm_tc_grouped(second, 2, status, st, 2, share));
     return BRISK_OK;
   }
   float* Hm = at<float>(ws, w.Hm);

@@ -323,8 +323,11 @@ struct TcSpec {
 };
 // `stages` (2 or 4) sets the shared-memory pipeline depth: 2 leaves room on each SM for other
 // kernels running concurrently.
+// small_carveout: the kernel (a separate instantiation) prefers the small shared-memory
+// carveout of the sweep, so that its CTAs can share SMs with sweep CTAs; the tiles must then fit
+// it (64-wide, two stages: 49 KB).
 cudaError_t gemm_tc_grouped(const TcSpec* spec, int nprob, int32_t* status, cudaStream_t stream,
-                            int stages);
+                            int stages, bool small_carveout = false);
 bool gemm_tc_supported(const void* A, int lda, const void* B, int ldb, int K);
 // dst[i*ldd + j] = (dst type) src[i*lds + j], i < rows, j < cols (src[j*lds + i] with transpose).
 cudaError_t copy2d(int rows, int cols, const void* src, int s_dt, int lds, void* dst, int d_dt,

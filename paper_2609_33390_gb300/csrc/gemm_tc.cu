@@ -172,7 +172,9 @@ struct TcArgs {
 constexpr int TC_OUT_CHUNK_F32 = TC_BM * 32 * 4;
 constexpr int TC_OUT_CHUNK_BF16X3 = 3 * TC_BM * 32 * 2;
 
-template <int TC_STAGES>
+// SMALL_CARVEOUT does not change the code: it makes a separate kernel whose shared-memory
+// carveout preference (a per-kernel attribute) is the sweep's.
+template <int TC_STAGES, bool SMALL_CARVEOUT = false>
 __global__ void __launch_bounds__(TC_THREADS, 1)
 gemm_tc_kernel(const __grid_constant__ TcMaps maps, const __grid_constant__ TcArgs a) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
@@ -417,8 +419,9 @@ bool gemm_tc_supported(const void* A, int lda, const void* B, int ldb, int K) {
 // One or two products C = A B^T, A [M, K] (row stride lda) and B [N, K] (row stride ldb) bf16,
 // fp32 accumulation, in one launch.
 cudaError_t gemm_tc_grouped(const TcSpec* spec, int nprob, int32_t* status, cudaStream_t stream,
-                            int stages) {
+                            int stages, bool small_carveout) {
   if (nprob < 1 || nprob > 2 || (stages != 2 && stages != 4)) return cudaErrorInvalidValue;
+  if (small_carveout && stages != 2) return cudaErrorInvalidValue;
   int nmax = 0;
   for (int i = 0; i < nprob; ++i) nmax = spec[i].N > nmax ? spec[i].N : nmax;
   if (spec[0].max_bn >= 16 && nmax > spec[0].max_bn) nmax = spec[0].max_bn;
@@ -459,11 +462,12 @@ cudaError_t gemm_tc_grouped(const TcSpec* spec, int nprob, int32_t* status, cuda
   }
   if (total == 0) return cudaSuccess;
   const size_t smem = gemm_tc_smem(BN, stages);
-  auto kernel = stages == 2 ? gemm_tc_kernel<2> : gemm_tc_kernel<4>;
+  if (small_carveout && smem > (size_t)(CARVEOUT_SMALL_KB - 1) * 1024) return cudaErrorInvalidValue;
+  auto kernel = small_carveout ? gemm_tc_kernel<2, true>
+                               : (stages == 2 ? gemm_tc_kernel<2> : gemm_tc_kernel<4>);
   cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(smem));
-  if (e == cudaSuccess) e = stages == 2 ? prefer_carveout(gemm_tc_kernel<2>, CARVEOUT_GEMM_KB)
-                                        : prefer_carveout(gemm_tc_kernel<4>, CARVEOUT_GEMM_KB);
+  if (e == cudaSuccess) e = prefer_carveout(kernel, small_carveout ? CARVEOUT_SMALL_KB : CARVEOUT_GEMM_KB);
   if (e != cudaSuccess) return e;
   e = launch_prio(kernel, dim3(total), dim3(TC_THREADS), smem, stream, maps, a);
   if (e != cudaSuccess) return e;
