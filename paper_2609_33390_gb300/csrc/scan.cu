@@ -830,28 +830,32 @@ corrector_kernel(const __grid_constant__ ScanArgs a) {
         gh4[m] = addc(gnh[m], pnh[m]);
       }
     }
-    // residual dots by a warp reduce-scatter; across warps through shared memory
-    float r = reduce_scatter_n<NP>(part);
+    // residual dots by a warp reduce-scatter; across warps through shared memory, where lane k
+    // sums the warps' partials of dot k (one shuffle fewer on the step's chain than summing in
+    // the reduce-scatter's lanes and moving dot k to lane k afterwards)
+    const float r = reduce_scatter_n<NP>(part);
     gacc = warp_sum(gacc);
-    if (NW > 1) {
+    float dk;
+    if constexpr (NW > 1) {
       float* red = sm.red + buf * NW * 32;
       if ((lane & (LSTEP - 1)) == 0) red[warp * 32 + lane / LSTEP] = r;
       if (lane == 0) sm.gpart[buf * NW + warp] = gacc;
       __syncthreads();
-      const int vidx = (lane / LSTEP) & (NP - 1);
-      r = red[vidx];
+      const int vidx = lane & (NP - 1);
+      dk = red[vidx];
       gacc = sm.gpart[buf * NW];
       for (int w = 1; w < NW; ++w) {
-        r += red[w * 32 + vidx];
+        dk += red[w * 32 + vidx];
         gacc += sm.gpart[buf * NW + w];
       }
+    } else {
+      dk = __shfl_sync(FULL_MASK, r, (lane * LSTEP) & 31);
     }
     // gate, refined scores (lane k: candidate k) and Select, identically in every warp
     float gate = a.b_g + gacc;
 #pragma unroll
     for (int f = 0; f < 5; ++f) gate = fmaf(wgf[f], phi[f], gate);
     const float gamma = sig_alpha * sigmoid_fast(gate);
-    const float dk = __shfl_sync(FULL_MASK, r, (lane * LSTEP) & 31);
     const float ref = lane < K ? sm.clp[i * K + lane] + gamma * dk : -INFINITY;
     const float u_cur_draw = u_cur;
     const int pick = select_warp(ref, K, a.select_mode, u_cur);
