@@ -547,10 +547,11 @@ __device__ __forceinline__ void gather_logits(const void* logits, int dt, int n,
 // keep them all in flight. Table rows are read through L2 (cache-global loads) a whole position
 // ahead into registers; an L2 line prefetch two positions ahead on top of that was slower
 // (single 105.7 -> 102.5 us for the products and the corrector without it, large_vocab
-// 269 -> 253 us). Shared memory holds only small per-sequence tables.
+// 269 -> 253 us). Shared memory holds the per-sequence tables (candidates, their log-probs, the
+// features' logits) and, for 4-element chunks, the feature shares and gate weights.
 // VERIFY: the CTA also verifies its sequence after the scan (the fused small-batch schedule); a
-// separate instantiation, since the verification code raises the scan's register count (123 ->
-// 164 a thread for four warps of 2-element chunks and K = 8), which would leave less room for
+// separate instantiation, since the verification code raises the scan's register count (122 ->
+// 143 a thread for four warps of 2-element chunks and K = 8), which would leave less room for
 // the verifier-row sweep beside the corrector in the overlapping schedule.
 template <int NW, int NP, int CMC, int CW, bool VERIFY>
 __global__ void __launch_bounds__(NW * 32)
