@@ -151,8 +151,9 @@ def test_unaligned_rows_and_base(brisk):
 
 def test_overlap_schedule_matches_unfused(brisk):
     """At least 2432 rows (one proposal-sweep task per row) take the overlapping schedule: the
-    verifier sweep from the start, 256-wide tiles for the hidden projection. Bit for bit the
-    same as the three separate calls (narrow tiles, serial), and parity with the oracle."""
+    verifier sweep from the start, the products in that schedule's tiles (2-stage, in the
+    sweep's carveout for this state width). Bit for bit the same as the three separate calls
+    (4-stage tiles, serial), and parity with the oracle."""
     wl = synth.Workload("overlap", B=80, L=32, V=4096, d=512, K=8, r=256)
     weights = _to(synth.make_weights(wl, "cpu"), "cuda")
     block = _to(synth.make_block(wl, "cpu"), "cuda")
